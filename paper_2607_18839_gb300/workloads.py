@@ -1,0 +1,239 @@
+"""Seeded synthetic inputs for one branch-decode step.
+
+This module only draws inputs.  It holds none of the step's arithmetic (no
+attention, no softmax, no argmax): it is the single input source shared by
+the CUDA path and the oracle.  Everything is numpy; bfloat16 tensors are kept
+as their uint16 bit patterns.
+
+Shapes follow the paper's pages (stand-ins for OmniDocBench pages, which are
+not available here): a page's shared prefix is its vision tokens plus the
+layout branch's tokens (Sec. 3.2 "Visual Encoder", Sec. 3.3), content
+branches fork from it, and each branch carries m P-MTP query tokens
+(Sec. 3.4).  Paged KV uses 16-token pages in a seeded random physical order.
+
+Presets ``c1`` .. ``c5`` are the five workloads of the branch-decode
+benchmark:
+
+c1  one page, prefix 256, 4 branches with suffix 8/16/24/32, m=1, H_q 8 / H_kv 2, D 64
+c2  one page, prefix 1,152 (1,024 vision + 128 layout), 16 branches with suffix
+    U[16,256], m=4, H_q 16 / H_kv 2, D 128
+c3  one page, prefix 4,096, 64 branches with suffix round(lognormal(4.5, 0.8))
+    clipped to [1, 1024], m=4, H_q 32 / H_kv 8, D 128
+c4  32 pages, prefix U[1024, 3072] each, 24 branches per page with lognormal
+    suffixes, m=8, H_q 16 / H_kv 2, D 128, one global page pool
+c5  one page, prefix 8,192, 256 branches with suffix
+    clip(floor(8 (1 + Pareto(1.5))), 8, 2048), m=4, H_q 32 / H_kv 8, D 128;
+    plus acceptance inputs: logits [256, 4, 32000] ~ N(0,1) in bf16
+
+"suffix" s_b is the private history already cached; the branch's private
+length is L_b = s_b + m because the step's own m tokens are written to the
+cache before attention.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import Optional
+
+import numpy as np
+
+PAGE = 16
+
+
+def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round float32 values to bfloat16 (round to nearest, ties to even)."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    bias = ((u >> 16) & 1) + 0x7FFF
+    return ((u + bias) >> 16).astype(np.uint16)
+
+
+def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
+    """Widen bfloat16 bit patterns to float32 (exact)."""
+    return (np.ascontiguousarray(b, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+@dataclass
+class BranchDecodeInputs:
+    """All inputs of one branch-attention call (host numpy arrays)."""
+
+    n_docs: int
+    B: int
+    m: int
+    H_q: int
+    H_kv: int
+    D: int
+    num_pages: int
+    max_pages: int
+    q: np.ndarray             # uint16 [B*m, H_q, D]
+    prefix_k: np.ndarray      # uint16 [sum P_d, H_kv, D]
+    prefix_v: np.ndarray
+    prefix_cu: np.ndarray     # int32 [n_docs+1]
+    branch_cu: np.ndarray     # int32 [n_docs+1]
+    k_cache: np.ndarray       # uint16 [num_pages, 16, H_kv, D]
+    v_cache: np.ndarray
+    page_table: np.ndarray    # int32 [B, max_pages]
+    branch_len: np.ndarray    # int32 [B]
+    branch_prefix_len: Optional[np.ndarray] = None  # int32 [B] or None
+    scale: float = 0.0        # 0 -> 1/sqrt(D)
+    name: str = "custom"
+    meta: dict = field(default_factory=dict)
+
+    @property
+    def rows(self) -> int:
+        return self.B * self.m
+
+    @property
+    def prefix_tokens(self) -> int:
+        return int(self.prefix_cu[-1])
+
+    @property
+    def max_prefix_len(self) -> int:
+        return int(np.max(np.diff(self.prefix_cu))) if self.n_docs else 0
+
+
+def _normal_bf16(rng: np.random.Generator, shape, std: float) -> np.ndarray:
+    return f32_to_bf16_bits(rng.standard_normal(shape, dtype=np.float32) * np.float32(std))
+
+
+def build_inputs(
+    prefix_lens,
+    branches_per_doc,
+    suffix_lens,
+    m: int,
+    H_q: int,
+    H_kv: int,
+    D: int,
+    seed: int,
+    *,
+    std: float = 0.5,
+    branch_prefix_len=None,
+    extra_pages: int = 0,
+    max_pages: Optional[int] = None,
+    scale: float = 0.0,
+    name: str = "custom",
+) -> BranchDecodeInputs:
+    """Draw one workload.
+
+    prefix_lens[d]       shared-prefix length P_d of page d
+    branches_per_doc[d]  number of content branches forked from page d
+    suffix_lens[b]       cached private history s_b of branch b (L_b = s_b + m)
+    branch_prefix_len    optional per-branch fork-position prefix (<= P_d)
+    extra_pages          unused pages mixed into the pool
+    """
+    rng = np.random.default_rng(seed)
+    prefix_lens = np.asarray(prefix_lens, dtype=np.int64)
+    branches_per_doc = np.asarray(branches_per_doc, dtype=np.int64)
+    n_docs = len(prefix_lens)
+    assert len(branches_per_doc) == n_docs
+    B = int(branches_per_doc.sum())
+    suffix_lens = np.asarray(suffix_lens, dtype=np.int64)
+    assert len(suffix_lens) == B
+    branch_len = (suffix_lens + m).astype(np.int32)
+    assert np.all(branch_len >= 0)
+
+    prefix_cu = np.zeros(n_docs + 1, dtype=np.int32)
+    prefix_cu[1:] = np.cumsum(prefix_lens)
+    branch_cu = np.zeros(n_docs + 1, dtype=np.int32)
+    branch_cu[1:] = np.cumsum(branches_per_doc)
+
+    pages_needed = (branch_len.astype(np.int64) + PAGE - 1) // PAGE
+    if max_pages is None:
+        max_pages = int(max(1, pages_needed.max() if B else 1))
+    assert np.all(pages_needed <= max_pages)
+    used = int(pages_needed.sum())
+    num_pages = max(1, used + extra_pages)
+    perm = rng.permutation(num_pages).astype(np.int32)
+
+    page_table = np.zeros((max(B, 0), max_pages), dtype=np.int32)
+    cursor = 0
+    for b in range(B):
+        n = int(pages_needed[b])
+        page_table[b, :n] = perm[cursor:cursor + n]
+        cursor += n
+        # entries past the branch's last page are never read; keep them valid ids
+        page_table[b, n:] = rng.integers(0, num_pages, size=max_pages - n)
+
+    T = int(prefix_cu[-1])
+    q = _normal_bf16(rng, (B * m, H_q, D), std)
+    prefix_k = _normal_bf16(rng, (T, H_kv, D), std)
+    prefix_v = _normal_bf16(rng, (T, H_kv, D), std)
+    k_cache = _normal_bf16(rng, (num_pages, PAGE, H_kv, D), std)
+    v_cache = _normal_bf16(rng, (num_pages, PAGE, H_kv, D), std)
+
+    bpl = None
+    if branch_prefix_len is not None:
+        bpl = np.asarray(branch_prefix_len, dtype=np.int32)
+        assert len(bpl) == B
+
+    return BranchDecodeInputs(
+        n_docs=n_docs, B=B, m=m, H_q=H_q, H_kv=H_kv, D=D, num_pages=num_pages,
+        max_pages=max_pages, q=q, prefix_k=prefix_k, prefix_v=prefix_v,
+        prefix_cu=prefix_cu, branch_cu=branch_cu, k_cache=k_cache, v_cache=v_cache,
+        page_table=page_table, branch_len=branch_len, branch_prefix_len=bpl,
+        scale=scale, name=name,
+        meta=dict(seed=seed, suffix_lens=suffix_lens.astype(np.int32)),
+    )
+
+
+def _lognormal_suffix(rng, n):
+    return np.clip(np.round(rng.lognormal(4.5, 0.8, size=n)), 1, 1024).astype(np.int64)
+
+
+def make_config(name: str, seed: Optional[int] = None) -> BranchDecodeInputs:
+    """One of the five preset workloads (see module docstring)."""
+    cid = int(name.lstrip("c"))
+    if seed is None:
+        seed = 1000 + cid
+    rng = np.random.default_rng(seed + 7919)  # lengths; tensors use ``seed``
+    if cid == 1:
+        return build_inputs([256], [4], [8, 16, 24, 32], 1, 8, 2, 64, seed, name="c1")
+    if cid == 2:
+        s = rng.integers(16, 257, size=16)
+        return build_inputs([1152], [16], s, 4, 16, 2, 128, seed, name="c2")
+    if cid == 3:
+        s = _lognormal_suffix(rng, 64)
+        return build_inputs([4096], [64], s, 4, 32, 8, 128, seed,
+                            max_pages=(1024 + 4 + PAGE - 1) // PAGE, name="c3")
+    if cid == 4:
+        P = rng.integers(1024, 3073, size=32)
+        s = _lognormal_suffix(rng, 32 * 24)
+        return build_inputs(P, [24] * 32, s, 8, 16, 2, 128, seed,
+                            max_pages=(1024 + 8 + PAGE - 1) // PAGE, name="c4")
+    if cid == 5:
+        s = np.clip(np.floor(8.0 * (1.0 + rng.pareto(1.5, size=256))), 8, 2048).astype(np.int64)
+        return build_inputs([8192], [256], s, 4, 32, 8, 128, seed,
+                            max_pages=(2048 + 4 + PAGE - 1) // PAGE, name="c5")
+    raise ValueError(f"unknown workload {name!r}")
+
+
+CONFIG_NAMES = ("c1", "c2", "c3", "c4", "c5")
+
+# Human-readable description of each preset, used in benchmark output.
+CONFIG_DESCRIPTIONS = {
+    "c1": "1 page, prefix 256, 4 branches (suffix 8/16/24/32), m=1, Hq8/Hkv2, D64",
+    "c2": "1 page, prefix 1152, 16 branches (suffix U[16,256]), m=4, Hq16/Hkv2, D128",
+    "c3": "1 page, prefix 4096, 64 branches (suffix lognormal(4.5,0.8)), m=4, Hq32/Hkv8, D128",
+    "c4": "32 pages, prefix U[1024,3072], 24 branches/page (lognormal), m=8, Hq16/Hkv2, D128",
+    "c5": "1 page, prefix 8192, 256 branches (suffix Pareto(1.5,min 8)<=2048), m=4, Hq32/Hkv8, D128",
+}
+
+
+def make_logits(B: int, m: int, V: int, seed: int) -> np.ndarray:
+    """bf16 logits [B, m, V] drawn N(0, 1)."""
+    rng = np.random.default_rng(seed)
+    return f32_to_bf16_bits(rng.standard_normal((B, m, V), dtype=np.float32))
+
+
+def mix_drafts(target_tokens: np.ndarray, V: int, p_match: float, seed: int) -> np.ndarray:
+    """Draft tokens: ``target_tokens`` (the caller's row argmax) with
+    probability ``p_match`` per position, else a uniform random token."""
+    rng = np.random.default_rng(seed)
+    target_tokens = np.asarray(target_tokens, dtype=np.int32)
+    keep = rng.random(target_tokens.shape) < p_match
+    rand = rng.integers(0, V, size=target_tokens.shape, dtype=np.int32)
+    return np.where(keep, target_tokens, rand).astype(np.int32)
+
+
+def accept_inputs(seed: int = 1005, B: int = 256, m: int = 4, V: int = 32000):
+    """Logits for the c5 acceptance step (drafts are mixed in by the caller
+    from the row argmax it trusts, via :func:`mix_drafts`)."""
+    return make_logits(B, m, V, seed)
