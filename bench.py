@@ -1,0 +1,512 @@
+#!/usr/bin/env python3
+"""Benchmark of the branch-decode step of Hierarchical Parallel Decoding.
+
+One step = one pass of the whole hot path over one batch of synthetic input:
+hpd_branch_attn (shared-prefix stage, private-suffix stage, LSE merge over the
+paged KV) followed by hpd_pmtp_accept (greedy verification of the P-MTP
+drafts against bf16 logits over a 32,000-token vocabulary).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c2]
+                    [--impl ours|reference]
+
+Prints ONE JSON line on rank 0.  The metric is query tokens (branches x m)
+per second; ``roofline`` reports the dominant kernel against the measured
+peaks in MEASURED_PEAKS.json; ``cpu_baseline`` times the fp64 oracle on the
+host cores.  ``--impl reference`` times the oracle itself as the bench arm.
+
+Timing: W warm-up steps, then exactly K steps replayed from CUDA graphs,
+bracketed by a barrier and a device synchronize, with the input replicas
+rotated so that their footprint exceeds 3x the L2 cache.  Per-kernel times
+come from timing markers recorded inside the graphs of the timed region.
+Under torchrun each rank processes its own pages (pages are independent; no
+collective on the data path) and the slowest rank's time is used.
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import glob
+import hashlib
+import io
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2607_18839_gb300 import workloads as W  # noqa: E402
+
+METRIC = "branch-decode query-tokens/s"
+UNIT = "query-tokens/s"
+VOCAB = 32000
+DRAFT_MATCH = 0.7
+KERNELS = ("prefix_stage", "suffix_stage", "lse_merge", "pmtp_accept")
+
+
+# ------------------------------------------------------------------ helpers --
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return dict(hbm=float(p["hbm_gbs"]), tc_burst=float(p["bf16_tflops"]),
+                    tc_sustained=float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                    source="measured")
+    return dict(hbm=6800.0, tc_burst=1900.0, tc_sustained=1700.0, source="fallback")
+
+
+def algorithmic_work(inp, V=VOCAB):
+    """Algorithmic bytes / FLOPs of one step, per kernel (the unit each
+    kernel must move or compute no matter how it is written)."""
+    m, Hq, Hkv, D = inp.m, inp.H_q, inp.H_kv, inp.D
+    P = np.diff(inp.prefix_cu).astype(np.float64)
+    Bd = np.diff(inp.branch_cu).astype(np.float64)
+    L = inp.branch_len.astype(np.float64)
+    rows = inp.B * m
+    q_bytes = rows * Hq * D * 2
+    prefix_kv = P.sum() * Hkv * D * 2 * 2
+    private_kv = L.sum() * Hkv * D * 2 * 2
+    pages_used = np.ceil(L / W.PAGE).sum()
+    tables = pages_used * 4 + inp.B * 4 + 2 * (inp.n_docs + 1) * 4
+    out_bytes = rows * Hq * D * 2 + rows * Hq * 4
+    prefix_flops = 4.0 * (Bd * m * Hq * P).sum() * D
+    vis = np.zeros(inp.B)
+    for i in range(m):
+        vis += np.maximum(0.0, L - m + i + 1)
+    suffix_flops = 4.0 * Hq * D * vis.sum()
+    accept_bytes = rows * V * 2 + rows * 4 * 2 + inp.B * 4
+    per = {
+        "prefix_stage": dict(bytes=prefix_kv + q_bytes, flops=prefix_flops),
+        "suffix_stage": dict(bytes=private_kv + q_bytes + tables, flops=suffix_flops),
+        "lse_merge": dict(bytes=out_bytes, flops=0.0),
+        "pmtp_accept": dict(bytes=accept_bytes, flops=0.0),
+    }
+    step_bytes = q_bytes + prefix_kv + private_kv + tables + out_bytes + accept_bytes
+    return per, dict(bytes=step_bytes, flops=prefix_flops + suffix_flops)
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2607_18839_gb300", "csrc", "*"))):
+        with open(p, "rb") as f:
+            h.update(os.path.basename(p).encode())
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(workload, kernel):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, or
+    None when there is none or the kernels changed since it was taken."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        t = json.load(f)
+    if t.get("kernel_source_hash") != kernel_source_hash():
+        return None
+    e = t.get("workloads", {}).get(workload, {}).get(kernel)
+    return None if e is None else float(e["dram_bytes_per_launch"])
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.15)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.1)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = [r for r in csv.reader(io.StringIO(out)) if len(r) >= 9]
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
+        smax = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for r in rows for k in range(4)
+                          if r[5 + k].strip().lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# ------------------------------------------------------------- CPU oracle --
+
+def oracle_sample_run(inp, logits, drafts, budget_s: float, rng_seed: int = 0):
+    """Time the fp64 oracle (attention + acceptance) on a bounded sample of
+    the workload: a random subset of branches, all their queries and heads,
+    repeated until ``budget_s`` seconds.  Returns (query tokens/s, threads,
+    sample description)."""
+    import oracle
+    per, _ = algorithmic_work(inp)
+    est_flops = 2.0 * (per["prefix_stage"]["flops"] + per["suffix_stage"]["flops"]) / inp.B
+    threads = oracle.max_threads()
+    per_branch_s = est_flops / (0.5e9 * threads)  # ~0.5 GFLOP/s per thread, fp64 scalar loops
+    n = int(max(1, min(inp.B, budget_s / 3.0 / max(per_branch_s, 1e-9))))
+    rng = np.random.default_rng(rng_seed)
+    sel = np.sort(rng.choice(inp.B, size=n, replace=False)).astype(np.int32)
+    rows = (sel[:, None] * inp.m + np.arange(inp.m)).reshape(-1)
+    lg = logits[sel]
+    dr = drafts[sel]
+    reps, t0 = 0, time.perf_counter()
+    while True:
+        oracle.branch_attn(inp, branch_sel=sel)
+        oracle.pmtp_accept(lg, dr)
+        reps += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s or reps >= 1000:
+            break
+    value = reps * len(rows) / el
+    sample = (f"{n} of {inp.B} branches ({len(rows)} query tokens, all heads, full prefix + "
+              f"suffix, + acceptance of their {len(rows)} logits rows) x {reps} reps in {el:.1f} s")
+    return value, threads, sample
+
+
+# --------------------------------------------------------------- our path --
+
+def run_ours(args, world, rank, local):
+    import torch
+    import torch.distributed as dist
+    from paper_2607_18839_gb300 import build as hpd_build
+    from paper_2607_18839_gb300 import hpd as H
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py: no CUDA device (the CUDA path has no CPU fallback)")
+    if world > 1:
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    hpd_build.build()
+    H.load()
+
+    cid = int(args.workload.lstrip("c"))
+    inp = W.make_config(args.workload, seed=1000 + cid + 100 * rank)
+    logits_np = W.make_logits(inp.B, inp.m, VOCAB, seed=2000 + cid + 100 * rank)
+    stream = torch.cuda.Stream(device=dev)
+    sh = int(stream.cuda_stream)
+
+    # ---- replicas: footprint > 3x L2 so timed steps read from HBM
+    base = H.DeviceInputs.from_host(inp, device=dev)
+    logits0 = torch.from_numpy(logits_np.view(np.int16)).to(dev).view(torch.bfloat16)
+    tensors = [base.q, base.prefix_k, base.prefix_v, base.k_cache, base.v_cache, base.page_table,
+               base.branch_len, base.prefix_cu, base.branch_cu, logits0]
+    rep_bytes = sum(t.numel() * t.element_size() for t in tensors)
+    l2 = int(getattr(torch.cuda.get_device_properties(dev), "L2_cache_size", 128 << 20))
+    free, _ = torch.cuda.mem_get_info(dev)
+    R = max(2, math.ceil(3 * l2 / rep_bytes))
+    R = int(min(R, 256, max(2, (free * 0.5) // rep_bytes)))
+
+    def clone_inputs(d):
+        return H.DeviceInputs(**{k: (v.clone() if isinstance(v, torch.Tensor) else v)
+                                 for k, v in d.__dict__.items()})
+
+    reps = [base] + [clone_inputs(base) for _ in range(R - 1)]
+    logits = [logits0] + [logits0.clone() for _ in range(R - 1)]
+    op = H.BranchAttn(base, stream=stream)
+    argsets = [H.make_args(d, op.out, op.lse, op.workspace, op.workspace.numel()) for d in reps]
+    n_launch = H.hpd_branch_attn_launches(argsets[0])
+    out_tokens = torch.empty((inp.B, inp.m), dtype=torch.int32, device=dev)
+    acc = torch.empty((inp.B,), dtype=torch.int32, device=dev)
+
+    # drafts: the row argmax (from this library's first acceptance call) kept
+    # with probability 0.7 per position, else a uniform random token
+    zeros = torch.zeros((inp.B, inp.m), dtype=torch.int32, device=dev)
+    with torch.cuda.stream(stream):
+        H.hpd_pmtp_accept(logits0.data_ptr(), zeros.data_ptr(), inp.B, inp.m, VOCAB,
+                          out_tokens.data_ptr(), acc.data_ptr(), sh)
+    stream.synchronize()
+    drafts_np = W.mix_drafts(out_tokens.cpu().numpy(), VOCAB, DRAFT_MATCH, seed=3000 + rank)
+    drafts = torch.from_numpy(drafts_np).to(dev)
+
+    def step(r, ev=None):
+        if ev is None:
+            H.hpd_branch_attn(argsets[r], sh)
+        else:
+            H.hpd_branch_attn_marked(argsets[r], sh, ev)
+        H.hpd_pmtp_accept(logits[r].data_ptr(), drafts.data_ptr(), inp.B, inp.m, VOCAB,
+                          out_tokens.data_ptr(), acc.data_ptr(), sh)
+
+    # ---- warm-up (eager), also sets the kernels' function attributes
+    with torch.cuda.stream(stream):
+        for i in range(max(args.warmup, 3)):
+            step(i % R)
+    stream.synchronize()
+    err = op.errors(stream)
+    if err:
+        raise SystemExit(f"bench.py: device error flags {err:#x}")
+
+    # ---- graphs of S steps, each step with timing markers
+    K = args.steps
+    S = max(1, min(K, args.graph_steps))
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(n_launch + 1)] for _ in range(S)]
+    with torch.cuda.stream(stream):
+        for row in events:
+            for e in row:
+                e.record(stream)  # creates the handle
+    stream.synchronize()
+    handles = [[int(e.cuda_event) for e in row] for row in events]
+
+    def capture(nsteps, offset, with_events, h2d=None, d2h=None):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(nsteps):
+                r = (offset + i) % R
+                if h2d is not None:
+                    h2d(r)
+                step(r, handles[i] if with_events else None)
+                if d2h is not None:
+                    d2h()
+        return g
+
+    g_main = capture(S, 0, True)
+    g_rem = capture(K % S, S, False) if K % S else None
+    n_main = K // S
+
+    def timed(gm, gr, nm):
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(nm):
+            gm.replay()
+        if gr is not None:
+            gr.replay()
+        t1.record(stream)
+        torch.cuda.synchronize(dev)
+        ms = t0.elapsed_time(t1)
+        if world > 1:
+            t = torch.tensor([ms], dtype=torch.float64, device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            dist.barrier()
+            ms = float(t.item())
+        return ms
+
+    gpu_id = str(torch.cuda.get_device_properties(dev).uuid)
+    gpu_id = gpu_id if gpu_id.startswith("GPU-") else f"GPU-{gpu_id}"
+    clocks = ClockSampler(gpu_id)
+    clocks.start()
+    total_ms = timed(g_main, g_rem, n_main)
+    clk = clocks.stop()
+
+    # per-kernel durations: markers of the last replay of the S-step graph
+    # (steps i and i+1 bracket step i's acceptance kernel)
+    per_kernel = {k: [] for k in KERNELS}
+    for i in range(S):
+        ev = events[i]
+        per_kernel["prefix_stage"].append(ev[0].elapsed_time(ev[1]))
+        per_kernel["suffix_stage"].append(ev[1].elapsed_time(ev[2]))
+        per_kernel["lse_merge"].append(ev[2].elapsed_time(ev[3]))
+        if i + 1 < S:
+            per_kernel["pmtp_accept"].append(ev[n_launch].elapsed_time(events[i + 1][0]))
+    kernel_ms = {k: (statistics.mean(v) if v else None) for k, v in per_kernel.items()}
+
+    # ---- end to end: pinned host inputs in, results out, every step
+    host_q = torch.from_numpy(inp.q.view(np.int16)).pin_memory()
+    host_meta = [torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).pin_memory()
+                 for a in (inp.page_table, inp.branch_len, inp.prefix_cu, inp.branch_cu)]
+    host_logits = torch.from_numpy(logits_np.view(np.int16)).pin_memory()
+    host_drafts = torch.from_numpy(drafts_np).pin_memory()
+    host_out = torch.empty(op.out.shape, dtype=torch.bfloat16).pin_memory()
+    host_lse = torch.empty(op.lse.shape, dtype=torch.float32).pin_memory()
+    host_tok = torch.empty(out_tokens.shape, dtype=torch.int32).pin_memory()
+    host_acc = torch.empty(acc.shape, dtype=torch.int32).pin_memory()
+
+    def h2d(r):
+        d = reps[r]
+        d.q.view(torch.int16).copy_(host_q, non_blocking=True)
+        for dst, src in zip((d.page_table, d.branch_len, d.prefix_cu, d.branch_cu), host_meta):
+            dst.copy_(src, non_blocking=True)
+        logits[r].view(torch.int16).copy_(host_logits, non_blocking=True)
+        drafts.copy_(host_drafts, non_blocking=True)
+
+    def d2h():
+        host_out.copy_(op.out, non_blocking=True)
+        host_lse.copy_(op.lse, non_blocking=True)
+        host_tok.copy_(out_tokens, non_blocking=True)
+        host_acc.copy_(acc, non_blocking=True)
+
+    h2d_bytes = sum(t.numel() * t.element_size()
+                    for t in [host_q, *host_meta, host_logits, host_drafts])
+    d2h_bytes = sum(t.numel() * t.element_size() for t in (host_out, host_lse, host_tok, host_acc))
+    ge_main = capture(S, 0, False, h2d, d2h)
+    ge_rem = capture(K % S, S, False, h2d, d2h) if K % S else None
+    e2e_ms = timed(ge_main, ge_rem, n_main)
+    err = op.errors(stream)
+    if err:
+        raise SystemExit(f"bench.py: device error flags {err:#x}")
+
+    # ---- CPU baseline: the oracle on this host's cores (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, thr, sample = oracle_sample_run(inp, logits_np, drafts_np, args.cpu_seconds)
+        cpu = {"value": v, "unit": UNIT, "cores": thr, "kind": "oracle", "sample": sample}
+
+    if world > 1:
+        dist.destroy_process_group()
+    if rank != 0:
+        return None
+
+    qtok = inp.B * inp.m
+    ms_step = total_ms / K
+    value = world * qtok / (ms_step * 1e-3)
+    e2e_value = world * qtok / (e2e_ms / K * 1e-3)
+
+    pk = peaks()
+    per, step_work = algorithmic_work(inp)
+    known = {k: v for k, v in kernel_ms.items() if v is not None}
+    dom = max(known, key=known.get)
+    dom_ms = known[dom]
+    if per[dom]["flops"] > 0 and dom == "prefix_stage":
+        achieved = per[dom]["flops"] / (dom_ms * 1e-3) / 1e12
+        roof = {"bound": "tensor", "achieved": achieved, "peak": pk["tc_sustained"],
+                "unit": "TFLOP/s"}
+    else:
+        achieved = per[dom]["bytes"] / (dom_ms * 1e-3) / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm"], "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = ncu_traffic(args.workload, dom)
+    roof["kernel"] = dom
+    roof["peak_source"] = pk["source"] + (" sustained bf16" if roof["bound"] == "tensor" else " HBM copy")
+    t_roof = max(step_work["bytes"] / (pk["hbm"] * 1e9), step_work["flops"] / (pk["tc_sustained"] * 1e12))
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {
+            "workload": f"{args.workload}: {W.CONFIG_DESCRIPTIONS[args.workload]}; acceptance "
+                        f"over bf16 logits [{inp.B} x {inp.m} x {VOCAB}]",
+            "query_tokens_per_step": qtok,
+            "l2": f"{R} rotating input replicas ({R * rep_bytes / 2**20:.0f} MiB > 3x L2 "
+                  f"{l2 / 2**20:.0f} MiB)",
+            "timing": f"CUDA graphs of {S} steps, events on the launch stream",
+            "parallelism": f"dp{world} (independent pages per GPU, no collective)",
+        },
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
+                "d2h_bytes_per_step": d2h_bytes,
+                "note": "q, page table, lengths, offsets, logits and drafts H2D from pinned "
+                        "host memory and out, lse, tokens, accepted lengths D2H every step; "
+                        "prefix KV and paged KV cache resident"},
+        "gpu_launches": K * (n_launch + 1),
+        "roofline": roof,
+        "step_roofline": {"bytes": step_work["bytes"], "flops": step_work["flops"],
+                          "t_roofline_us": t_roof * 1e6,
+                          "frac": t_roof / (ms_step * 1e-3)},
+        "kernel_us": {k: (v * 1e3 if v is not None else None) for k, v in kernel_ms.items()},
+        "cpu_baseline": cpu,
+        "clocks": clk,
+    }
+    return line
+
+
+# --------------------------------------------------------- reference arm --
+
+def run_reference(args, world, rank):
+    """The fp64 oracle as the bench arm: each step runs it on a bounded
+    sample of the workload on this host's cores."""
+    if world > 1 and rank != 0:
+        return None
+    import oracle
+    inp = W.make_config(args.workload)
+    cid = int(args.workload.lstrip("c"))
+    logits = W.make_logits(inp.B, inp.m, VOCAB, seed=2000 + cid)
+    tok, _ = oracle.pmtp_accept(logits, np.zeros((inp.B, inp.m), np.int32))
+    drafts = W.mix_drafts(tok, VOCAB, DRAFT_MATCH, seed=3000)
+    per, _ = algorithmic_work(inp)
+    threads = oracle.max_threads()
+    est = 2.0 * (per["prefix_stage"]["flops"] + per["suffix_stage"]["flops"]) / inp.B
+    n = int(max(1, min(inp.B, args.ref_step_seconds / max(est / (0.5e9 * threads), 1e-9))))
+    rng = np.random.default_rng(0)
+    sel = np.sort(rng.choice(inp.B, size=n, replace=False)).astype(np.int32)
+    lg, dr = logits[sel], drafts[sel]
+    qtok = n * inp.m
+
+    def step():
+        oracle.branch_attn(inp, branch_sel=sel)
+        oracle.pmtp_accept(lg, dr)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    el = time.perf_counter() - t0
+    value = args.steps * qtok / el
+    sample = f"{n} of {inp.B} branches ({qtok} query tokens, all heads) + their acceptance rows per step"
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": f"{args.workload}: {W.CONFIG_DESCRIPTIONS[args.workload]}; acceptance "
+                               f"over bf16 logits [{inp.B} x {inp.m} x {VOCAB}]",
+                   "parallelism": "host CPU (OpenMP)"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--workload", choices=W.CONFIG_NAMES, default="c2")
+    ap.add_argument("--graph-steps", type=int, default=200, help="steps captured per CUDA graph")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle CPU-baseline budget")
+    ap.add_argument("--ref-step-seconds", type=float, default=1.0,
+                    help="oracle work per step of --impl reference")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world, rank, local = dist_env()
+    if args.impl == "reference":
+        line = run_reference(args, world, rank)
+    else:
+        line = run_ours(args, world, rank, local)
+    if line is not None and rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

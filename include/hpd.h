@@ -1,0 +1,174 @@
+/*
+ * hpd.h -- C ABI of libhpd, the GB300 (sm_103a) branch-decode step of
+ * Hierarchical Parallel Decoding (HPD-Parsing).
+ *
+ * One call of hpd_branch_attn is the attention of one decoder layer for one
+ * decode step of many concurrent content branches.  A content branch is
+ * forked from the layout branch of its page and attends to
+ *   - the page's shared prefix (the vision tokens plus the layout branch's
+ *     tokens up to the fork position), whose KV is reused, never recomputed,
+ *     and
+ *   - its own private KV history only, never that of another branch
+ * (Sec. 3.3, "Dynamic Branch Forking and Efficient Context Isolation").
+ * Each branch carries m P-MTP query tokens that are causal among themselves
+ * (Sec. 3.4, "Integration with P-MTP").  hpd_pmtp_accept is the greedy
+ * verification of the P-MTP drafts that follows the forward pass (Sec. 3.4;
+ * the verification step of Algorithm 1).
+ *
+ * Conventions for every entry point
+ *   - Every pointer named in an argument list or struct is DEVICE memory of
+ *     the current device, owned by the caller; the library keeps no pointer
+ *     after the call returns.  Nothing here allocates, frees or synchronises
+ *     (except hpd_read_errors, which says so).
+ *   - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream) and runs asynchronously.
+ *   - Host-side scalars are validated before anything is launched; a bad
+ *     value returns HPD_ERR_INVALID_ARG / HPD_ERR_UNSUPPORTED and launches
+ *     nothing.  Device-side integer arrays (offsets, lengths, page ids) are
+ *     not read by the host: the kernels clamp every such value into range
+ *     and record what they clamped in the workspace's error word (see
+ *     hpd_read_errors), so no device content can make a kernel access memory
+ *     outside the buffers described here.
+ *   - A failed launch returns HPD_ERR_CUDA; hpd_last_cuda_error() gives the
+ *     CUDA error code of the most recent failure on the calling thread.
+ *   - bf16 means IEEE bfloat16, stored as 2-byte little-endian words.
+ */
+#ifndef HPD_H_
+#define HPD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *hpd_stream_t; /* identical to cudaStream_t */
+
+typedef enum {
+  HPD_OK = 0,
+  HPD_ERR_INVALID_ARG = 1, /* a host scalar or pointer is out of contract */
+  HPD_ERR_UNSUPPORTED = 2, /* a legal shape this build has no kernel for */
+  HPD_ERR_WORKSPACE = 3,   /* workspace missing, misaligned or too small */
+  HPD_ERR_CUDA = 4,        /* a CUDA runtime call or launch failed */
+  HPD_ERR_TIMEOUT = 5      /* a bounded device-side wait gave up */
+} hpd_status;
+
+/* Bits of the workspace error word (sticky until hpd_workspace_init). */
+#define HPD_DEVERR_PREFIX_CU 0x1u   /* prefix_cu not monotone / beyond prefix_tokens */
+#define HPD_DEVERR_BRANCH_CU 0x2u   /* branch_cu not monotone / beyond B */
+#define HPD_DEVERR_BRANCH_LEN 0x4u  /* branch_len < 0 or > 16 * max_pages_per_branch */
+#define HPD_DEVERR_PAGE_ID 0x8u     /* a page id outside [0, num_pages) */
+#define HPD_DEVERR_FORK_LEN 0x10u   /* branch_prefix_len < 0 or > P_d */
+#define HPD_DEVERR_TIMEOUT 0x40u    /* a bounded device-side wait expired */
+
+/* Tokens per KV page of the paged private cache. */
+#define HPD_PAGE_TOKENS 16
+
+/*
+ * Arguments of one branch-attention step.
+ *
+ * Notation: n_docs pages (documents); page d owns branches
+ * [branch_cu[d], branch_cu[d+1]) and the prefix tokens
+ * [prefix_cu[d], prefix_cu[d+1]) of prefix_k / prefix_v, so P_d =
+ * prefix_cu[d+1] - prefix_cu[d].  Branch b has L_b = branch_len[b] private
+ * KV entries, which INCLUDE the K/V of this step's m query tokens (they are
+ * written to the cache before the call).  G = H_q / H_kv query heads share
+ * one KV head; query head h reads KV head h / G.
+ *
+ * Query i (0 <= i < m) of branch b sees
+ *   prefix keys  j <  P_b   (P_b = branch_prefix_len[b] if given, else P_d)
+ *   private keys j <= L_b - m + i
+ * Private key j is slot j % 16 of physical page page_table[b][j / 16].
+ * S_j = scale * <q, k_j>; out = softmax(S) V over the visible keys;
+ * lse = ln sum_j exp(S_j).  No visible key: out = 0, lse = -inf.
+ */
+typedef struct {
+  const void *q;        /* bf16 [B*m][H_q][D]; row b*m + i                        */
+  const void *prefix_k; /* bf16 [prefix_tokens][H_kv][D]                          */
+  const void *prefix_v; /* bf16 [prefix_tokens][H_kv][D]                          */
+  const int32_t *prefix_cu;         /* [n_docs+1], non-decreasing, <= prefix_tokens */
+  const int32_t *branch_cu;         /* [n_docs+1], non-decreasing, branch_cu[n_docs] == B */
+  const int32_t *branch_prefix_len; /* [B] fork-position prefix length, or NULL     */
+  const void *k_cache;  /* bf16 [num_pages][16][H_kv][D]                           */
+  const void *v_cache;  /* bf16 [num_pages][16][H_kv][D]                           */
+  const int32_t *page_table;        /* [B][max_pages_per_branch]                    */
+  const int32_t *branch_len;        /* [B], 0 <= L_b <= 16 * max_pages_per_branch   */
+  int n_docs;               /* >= 1                                               */
+  int B;                    /* >= 1 branches                                      */
+  int m;                    /* 1..16 P-MTP query tokens per branch                */
+  int H_q, H_kv;            /* H_q % H_kv == 0, G = H_q / H_kv <= 16               */
+  int D;                    /* head dim: 64 or 128                                */
+  int num_pages;            /* >= 1 pages in k_cache / v_cache                    */
+  int max_pages_per_branch; /* >= 1 columns of page_table                         */
+  int prefix_tokens;        /* rows of prefix_k / prefix_v (>= 0)                 */
+  int max_prefix_len;       /* host upper bound on every P_d; 0 = prefix_tokens   */
+  float scale;              /* softmax scale; 0 = 1/sqrt(D)                       */
+  void *out;                /* bf16 [B*m][H_q][D]                                 */
+  float *lse;               /* fp32 [B*m][H_q], natural log; may be NULL          */
+  void *workspace;          /* 256-byte aligned, initialised once by
+                               hpd_workspace_init; one call at a time per workspace */
+  size_t workspace_bytes;
+} hpd_branch_attn_args;
+
+/* Bytes of workspace hpd_branch_attn needs for these host scalars (the
+ * device pointers in args are not read).  Returns 0 if the scalars are
+ * invalid. */
+size_t hpd_branch_attn_workspace_size(const hpd_branch_attn_args *args);
+
+/* Zero the workspace (error word and internal counters) on `stream`.  Call
+ * once after allocating it; hpd_branch_attn leaves it reusable. */
+hpd_status hpd_workspace_init(void *workspace, size_t workspace_bytes, hpd_stream_t stream);
+
+/* The branch-decode attention step (see the struct above).  Enqueues its
+ * kernels on `stream`; out / lse are complete when the stream reaches that
+ * point.  Concurrent calls must use distinct workspaces. */
+hpd_status hpd_branch_attn(const hpd_branch_attn_args *args, hpd_stream_t stream);
+
+/* Number of kernels one hpd_branch_attn call launches for these scalars
+ * (0 if they are invalid): the shared-prefix stage, the private-suffix stage
+ * and the log-sum-exp merge, in that order. */
+int hpd_branch_attn_launches(const hpd_branch_attn_args *args);
+
+/* hpd_branch_attn with timing markers.  stage_events holds
+ * hpd_branch_attn_launches(args) + 1 cudaEvent_t handles created by the
+ * caller (with timing enabled); event 0 is recorded on `stream` before the
+ * first kernel and event k after the k-th.  Recorded as external events, so
+ * they also work inside stream capture.  NULL behaves as hpd_branch_attn. */
+hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *args, hpd_stream_t stream,
+                                  void *const *stage_events);
+
+/*
+ * Greedy P-MTP verification (Sec. 3.4; Algorithm 1, verification step).
+ *   logits       bf16 [B][m][V]   target-model logits at the m draft positions
+ *   drafts       int32 [B][m]     drafted tokens; drafts[b][j] is checked
+ *                                 against the argmax of logits row j
+ *   out_tokens   int32 [B][m]     t*_{b,j} = argmax_v logits[b][j][v], the
+ *                                 lowest index among equal maxima; NaN never
+ *                                 wins (an all-NaN row gives 0)
+ *   accepted_len int32 [B]        n_acc_b = largest k <= m such that
+ *                                 drafts[b][i] == t*_{b,i} for all i < k
+ * The caller emits t*_{b,0 .. min(n_acc_b, m-1)}: the accepted drafts plus
+ * the target's own token at the first mismatch.
+ * Requires B >= 1, 1 <= m <= 64, V >= 1.
+ */
+hpd_status hpd_pmtp_accept(const void *logits, const int32_t *drafts, int B, int m, int V,
+                           int32_t *out_tokens, int32_t *accepted_len, hpd_stream_t stream);
+
+/* Copy the workspace error word (HPD_DEVERR_* bits) to *flags.  This is the
+ * one call that synchronises: it waits for `stream`. */
+hpd_status hpd_read_errors(const void *workspace, uint32_t *flags, hpd_stream_t stream);
+
+/* Static description of a status code. */
+const char *hpd_status_string(hpd_status status);
+
+/* CUDA error code (cudaError_t value) of the last HPD_ERR_CUDA on this thread. */
+int hpd_last_cuda_error(void);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int hpd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* HPD_H_ */

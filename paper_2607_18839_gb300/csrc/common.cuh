@@ -1,0 +1,128 @@
+// common.cuh -- device helpers and the internal plan shared by libhpd's kernels.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/hpd.h"
+
+namespace hpd {
+
+constexpr int kPage = HPD_PAGE_TOKENS;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+// ---------------------------------------------------------------- plan --
+// Host-computed launch plan of one hpd_branch_attn call.  Only host scalars
+// enter it, so it can be computed before any device data is known.
+struct Plan {
+  int G;           // query heads per KV head
+  int rows_total;  // B * m query tokens
+  int S_p;         // key splits of the shared prefix per row tile
+  int S_s;         // key splits of a branch's private suffix
+  int tiles_max;   // upper bound of prefix row tiles per KV head
+  int wr_s;        // warps along rows in the suffix kernel (1, 2, 4)
+  int rt_s;        // suffix row tiles per (branch, KV head)
+  size_t off_err;    // uint32 error word
+  size_t off_opart;  // fp32 [S_p + S_s][rows_total][H_q][D]
+  size_t off_lpart;  // fp32 [S_p + S_s][rows_total][H_q]
+  size_t bytes;      // total workspace bytes
+};
+
+// Kernel parameters of the two attention stages (prefix and suffix).
+struct AttnParams {
+  const __nv_bfloat16 *q;
+  const __nv_bfloat16 *prefix_k;
+  const __nv_bfloat16 *prefix_v;
+  const int32_t *prefix_cu;
+  const int32_t *branch_cu;
+  const int32_t *branch_prefix_len;
+  const __nv_bfloat16 *k_cache;
+  const __nv_bfloat16 *v_cache;
+  const int32_t *page_table;
+  const int32_t *branch_len;
+  int n_docs, B, m, H_q, H_kv, G, D;
+  int num_pages, max_pages, prefix_tokens;
+  float scale_log2;  // softmax scale * log2(e)
+  int S_p, S_s, rows_total;
+  float *o_part;
+  float *l_part;
+  uint32_t *err;
+};
+
+// Kernel parameters of the merge stage.
+struct MergeParams {
+  const float *o_part;
+  const float *l_part;
+  int S_total, rows_total, H_q, D;
+  __nv_bfloat16 *out;
+  float *lse;
+};
+
+// ------------------------------------------------------- device helpers --
+__device__ __forceinline__ void flag_error(uint32_t *err, uint32_t bit) {
+  if (err) atomicOr(err, bit);
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// 16-byte async global->shared copy; src_bytes == 0 writes zeros.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, int src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src),
+               "r"(src_bytes));
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N));
+}
+
+__device__ __forceinline__ void ldmatrix_x4(uint32_t addr, uint32_t &r0, uint32_t &r1,
+                                            uint32_t &r2, uint32_t &r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t addr, uint32_t &r0, uint32_t &r1,
+                                                  uint32_t &r2, uint32_t &r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+// D(16x8, fp32) += A(16x16, bf16, row) * B(16x8, bf16, col)
+__device__ __forceinline__ void mma_bf16_16816(float *d, const uint32_t *a, uint32_t b0,
+                                               uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t *>(&v);
+}
+
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;\n" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ int ceil_div_i(int a, int b) { return (a + b - 1) / b; }
+
+}  // namespace hpd
+
+// Host-side launchers (defined in the .cu files, called by hpd_api.cu).
+namespace hpd {
+cudaError_t launch_prefix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
+cudaError_t launch_suffix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
+cudaError_t launch_merge(const MergeParams &p, cudaStream_t s);
+cudaError_t launch_accept(const __nv_bfloat16 *logits, const int32_t *drafts, int B, int m, int V,
+                          int32_t *out_tokens, int32_t *accepted_len, cudaStream_t s);
+}  // namespace hpd

@@ -1,0 +1,213 @@
+// hpd_api.cu -- the C ABI of libhpd (include/hpd.h): host-side validation,
+// the launch plan and the workspace layout.  Every compute step runs in the
+// kernels of attn_mma.cu and merge_accept.cu; nothing here touches device
+// data.
+#include <cmath>
+#include <cstdint>
+
+#include "common.cuh"
+
+namespace {
+
+thread_local int g_last_cuda_error = 0;
+
+hpd_status cuda_fail(cudaError_t e) {
+  g_last_cuda_error = static_cast<int>(e);
+  return HPD_ERR_CUDA;
+}
+
+constexpr size_t kAlign = 256;
+constexpr int kPrefixTileRows = 64;   // rows per prefix-stage CTA
+constexpr int kTargetCtas = 152 * 4;  // prefix-stage CTAs aimed for (GB300: 152 SMs)
+constexpr int kMaxPrefixSplits = 16;
+constexpr int kSuffixSplitKeys = 1024;  // a suffix chunk holds at most ~this many keys
+constexpr int kMaxSuffixSplits = 8;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+int ceil_div(long long a, long long b) { return static_cast<int>((a + b - 1) / b); }
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Host-scalar checks shared by the workspace query and the call itself.
+hpd_status check_scalars(const hpd_branch_attn_args *a) {
+  if (!a) return HPD_ERR_INVALID_ARG;
+  if (a->n_docs < 1 || a->B < 1 || a->m < 1 || a->H_q < 1 || a->H_kv < 1 || a->num_pages < 1 ||
+      a->max_pages_per_branch < 1 || a->prefix_tokens < 0 || a->max_prefix_len < 0)
+    return HPD_ERR_INVALID_ARG;
+  if (a->m > 16) return HPD_ERR_UNSUPPORTED;
+  if (a->H_q % a->H_kv != 0) return HPD_ERR_INVALID_ARG;
+  if (a->H_q / a->H_kv > 16) return HPD_ERR_UNSUPPORTED;
+  if (a->D != 64 && a->D != 128) return HPD_ERR_UNSUPPORTED;
+  if (!std::isfinite(a->scale)) return HPD_ERR_INVALID_ARG;
+  const long long rows = static_cast<long long>(a->B) * a->m;
+  if (rows * a->H_q * a->D >= (1LL << 31)) return HPD_ERR_UNSUPPORTED;
+  if (static_cast<long long>(a->max_pages_per_branch) * hpd::kPage >= (1LL << 30))
+    return HPD_ERR_UNSUPPORTED;
+  return HPD_OK;
+}
+
+hpd::Plan make_plan(const hpd_branch_attn_args *a) {
+  hpd::Plan pl{};
+  pl.G = a->H_q / a->H_kv;
+  pl.rows_total = a->B * a->m;
+  const long long stacked = static_cast<long long>(a->B) * a->m * pl.G;
+  const int tiles = ceil_div(stacked, kPrefixTileRows);
+  pl.tiles_max = tiles + a->n_docs;
+  const int maxP = a->max_prefix_len > 0 ? std::min(a->max_prefix_len, a->prefix_tokens)
+                                         : a->prefix_tokens;
+  const long long tiles_est = static_cast<long long>(std::max(tiles, 1)) * a->H_kv;
+  int sp = ceil_div(kTargetCtas, tiles_est);
+  sp = std::min(sp, std::max(1, ceil_div(maxP, 256)));
+  pl.S_p = std::max(1, std::min(sp, kMaxPrefixSplits));
+  const int maxL = a->max_pages_per_branch * hpd::kPage;
+  pl.S_s = std::max(1, std::min(ceil_div(maxL, kSuffixSplitKeys), kMaxSuffixSplits));
+  const int rows_s = a->m * pl.G;
+  pl.wr_s = rows_s <= 16 ? 1 : (rows_s <= 32 ? 2 : 4);
+  pl.rt_s = ceil_div(rows_s, 16 * pl.wr_s);
+  const size_t S = static_cast<size_t>(pl.S_p + pl.S_s);
+  const size_t pairs = static_cast<size_t>(pl.rows_total) * a->H_q;
+  pl.off_err = 0;
+  pl.off_opart = kAlign;
+  pl.off_lpart = align_up(pl.off_opart + S * pairs * a->D * sizeof(float));
+  pl.bytes = align_up(pl.off_lpart + S * pairs * sizeof(float));
+  return pl;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t hpd_branch_attn_workspace_size(const hpd_branch_attn_args *args) {
+  if (check_scalars(args) != HPD_OK) return 0;
+  return make_plan(args).bytes;
+}
+
+hpd_status hpd_workspace_init(void *workspace, size_t workspace_bytes, hpd_stream_t stream) {
+  if (!workspace || !aligned(workspace, kAlign) || workspace_bytes < kAlign)
+    return HPD_ERR_WORKSPACE;
+  const cudaError_t e = cudaMemsetAsync(workspace, 0, kAlign, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? HPD_OK : cuda_fail(e);
+}
+
+int hpd_branch_attn_launches(const hpd_branch_attn_args *args) {
+  return check_scalars(args) == HPD_OK ? 3 : 0;
+}
+
+hpd_status hpd_branch_attn(const hpd_branch_attn_args *a, hpd_stream_t stream) {
+  return hpd_branch_attn_marked(a, stream, nullptr);
+}
+
+hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t stream,
+                                  void *const *ev) {
+  const hpd_status st = check_scalars(a);
+  if (st != HPD_OK) return st;
+  if (!a->q || !a->prefix_cu || !a->branch_cu || !a->k_cache || !a->v_cache || !a->page_table ||
+      !a->branch_len || !a->out)
+    return HPD_ERR_INVALID_ARG;
+  if (a->prefix_tokens > 0 && (!a->prefix_k || !a->prefix_v)) return HPD_ERR_INVALID_ARG;
+  if (!aligned(a->q, 16) || !aligned(a->prefix_k, 16) || !aligned(a->prefix_v, 16) ||
+      !aligned(a->k_cache, 16) || !aligned(a->v_cache, 16) || !aligned(a->out, 16) ||
+      !aligned(a->lse, 4) || !aligned(a->prefix_cu, 4) || !aligned(a->branch_cu, 4) ||
+      !aligned(a->page_table, 4) || !aligned(a->branch_len, 4) ||
+      !aligned(a->branch_prefix_len, 4))
+    return HPD_ERR_INVALID_ARG;
+  const hpd::Plan pl = make_plan(a);
+  if (!a->workspace || !aligned(a->workspace, kAlign) || a->workspace_bytes < pl.bytes)
+    return HPD_ERR_WORKSPACE;
+
+  uint8_t *ws = static_cast<uint8_t *>(a->workspace);
+  hpd::AttnParams p{};
+  p.q = static_cast<const __nv_bfloat16 *>(a->q);
+  p.prefix_k = static_cast<const __nv_bfloat16 *>(a->prefix_k ? a->prefix_k : a->k_cache);
+  p.prefix_v = static_cast<const __nv_bfloat16 *>(a->prefix_v ? a->prefix_v : a->v_cache);
+  p.prefix_cu = a->prefix_cu;
+  p.branch_cu = a->branch_cu;
+  p.branch_prefix_len = a->branch_prefix_len;
+  p.k_cache = static_cast<const __nv_bfloat16 *>(a->k_cache);
+  p.v_cache = static_cast<const __nv_bfloat16 *>(a->v_cache);
+  p.page_table = a->page_table;
+  p.branch_len = a->branch_len;
+  p.n_docs = a->n_docs;
+  p.B = a->B;
+  p.m = a->m;
+  p.H_q = a->H_q;
+  p.H_kv = a->H_kv;
+  p.G = pl.G;
+  p.D = a->D;
+  p.num_pages = a->num_pages;
+  p.max_pages = a->max_pages_per_branch;
+  p.prefix_tokens = a->prefix_tokens;
+  const float scale = a->scale != 0.f ? a->scale : 1.0f / std::sqrt(static_cast<float>(a->D));
+  p.scale_log2 = scale * hpd::kLog2e;
+  p.S_p = pl.S_p;
+  p.S_s = pl.S_s;
+  p.rows_total = pl.rows_total;
+  p.o_part = reinterpret_cast<float *>(ws + pl.off_opart);
+  p.l_part = reinterpret_cast<float *>(ws + pl.off_lpart);
+  p.err = reinterpret_cast<uint32_t *>(ws + pl.off_err);
+
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  auto mark = [&](int k) -> cudaError_t {
+    if (!ev || !ev[k]) return cudaSuccess;
+    return cudaEventRecordWithFlags(static_cast<cudaEvent_t>(ev[k]), s, cudaEventRecordExternal);
+  };
+  cudaError_t e = mark(0);
+  if (e == cudaSuccess) e = hpd::launch_prefix_stage(p, pl, s);
+  if (e == cudaSuccess) e = mark(1);
+  if (e == cudaSuccess) e = hpd::launch_suffix_stage(p, pl, s);
+  if (e == cudaSuccess) e = mark(2);
+  if (e != cudaSuccess) return cuda_fail(e);
+
+  hpd::MergeParams mp{};
+  mp.o_part = p.o_part;
+  mp.l_part = p.l_part;
+  mp.S_total = pl.S_p + pl.S_s;
+  mp.rows_total = pl.rows_total;
+  mp.H_q = a->H_q;
+  mp.D = a->D;
+  mp.out = static_cast<__nv_bfloat16 *>(a->out);
+  mp.lse = a->lse;
+  e = hpd::launch_merge(mp, s);
+  if (e == cudaSuccess) e = mark(3);
+  if (e != cudaSuccess) return cuda_fail(e);
+  return HPD_OK;
+}
+
+hpd_status hpd_pmtp_accept(const void *logits, const int32_t *drafts, int B, int m, int V,
+                           int32_t *out_tokens, int32_t *accepted_len, hpd_stream_t stream) {
+  if (!logits || !drafts || !out_tokens || !accepted_len) return HPD_ERR_INVALID_ARG;
+  if (B < 1 || m < 1 || V < 1) return HPD_ERR_INVALID_ARG;
+  if (m > 64) return HPD_ERR_UNSUPPORTED;
+  if (!aligned(logits, 2) || !aligned(drafts, 4) || !aligned(out_tokens, 4) ||
+      !aligned(accepted_len, 4))
+    return HPD_ERR_INVALID_ARG;
+  const cudaError_t e =
+      hpd::launch_accept(static_cast<const __nv_bfloat16 *>(logits), drafts, B, m, V, out_tokens,
+                         accepted_len, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? HPD_OK : cuda_fail(e);
+}
+
+hpd_status hpd_read_errors(const void *workspace, uint32_t *flags, hpd_stream_t stream) {
+  if (!workspace || !flags || !aligned(workspace, kAlign)) return HPD_ERR_INVALID_ARG;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemcpyAsync(flags, workspace, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  return e == cudaSuccess ? HPD_OK : cuda_fail(e);
+}
+
+const char *hpd_status_string(hpd_status status) {
+  switch (status) {
+    case HPD_OK: return "ok";
+    case HPD_ERR_INVALID_ARG: return "invalid argument";
+    case HPD_ERR_UNSUPPORTED: return "unsupported shape";
+    case HPD_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case HPD_ERR_CUDA: return "CUDA error";
+    case HPD_ERR_TIMEOUT: return "device-side wait timed out";
+  }
+  return "unknown status";
+}
+
+int hpd_last_cuda_error(void) { return g_last_cuda_error; }
+
+int hpd_version(void) { return 100; }
+
+}  // extern "C"

@@ -1,0 +1,88 @@
+"""The C-ABI library builds for sm_103a, loads, exports every entry point that
+include/hpd.h declares, and rejects bad host arguments before touching the
+GPU.  No compute call is made here, so these run without a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2607_18839_gb300 import build as B
+from paper_2607_18839_gb300 import hpd
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "hpd.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return hpd.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(hpd_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_every_declared_entry_point_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 8
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in include/hpd.h but not exported"
+    assert set(names) == set(hpd.EXPORTS)
+
+
+def test_version_and_status_strings(lib):
+    assert hpd.hpd_version() >= 100
+    assert hpd.hpd_status_string(0) == "ok"
+    assert "workspace" in hpd.hpd_status_string(3)
+
+
+def test_struct_layout_matches_c():
+    # 10 pointers, 10 ints, a float, 3 pointers and a size_t (x86_64 / aarch64)
+    assert ctypes.sizeof(hpd.hpd_branch_attn_args) == 80 + 40 + 8 + 24 + 8
+    assert hpd.hpd_branch_attn_args.out.offset == 128
+
+
+def _args(**kw):
+    a = hpd.hpd_branch_attn_args()
+    base = dict(n_docs=1, B=4, m=4, H_q=16, H_kv=2, D=128, num_pages=10,
+                max_pages_per_branch=4, prefix_tokens=100, max_prefix_len=0, scale=0.0)
+    base.update(kw)
+    for k, v in base.items():
+        setattr(a, k, v)
+    return a
+
+
+def test_workspace_size_rejects_bad_scalars(lib):
+    assert hpd.hpd_branch_attn_workspace_size(_args()) > 0
+    for bad in (dict(D=96), dict(H_q=15), dict(m=0), dict(m=17), dict(B=0), dict(n_docs=0),
+                dict(H_q=64, H_kv=2), dict(num_pages=0), dict(max_pages_per_branch=0),
+                dict(scale=float("nan"))):
+        assert hpd.hpd_branch_attn_workspace_size(_args(**bad)) == 0, bad
+
+
+def test_workspace_size_grows_with_rows(lib):
+    a = hpd.hpd_branch_attn_workspace_size(_args(B=4))
+    b = hpd.hpd_branch_attn_workspace_size(_args(B=64))
+    assert b > a > 0
+
+
+def test_branch_attn_rejects_bad_arguments_before_launch(lib):
+    # null device pointers are refused on the host: nothing is launched
+    with pytest.raises(hpd.HpdError) as e:
+        hpd.hpd_branch_attn(_args(), None)
+    assert e.value.status == 1
+    with pytest.raises(hpd.HpdError) as e:
+        hpd.hpd_branch_attn(_args(D=80), None)
+    assert e.value.status == 2
+
+
+def test_accept_rejects_bad_arguments_before_launch(lib):
+    with pytest.raises(hpd.HpdError) as e:
+        hpd.hpd_pmtp_accept(None, None, 4, 4, 100, None, None, None)
+    assert e.value.status == 1
+    with pytest.raises(hpd.HpdError) as e:
+        hpd.hpd_pmtp_accept(16, 16, 4, 65, 100, 16, 16, None)
+    assert e.value.status == 2

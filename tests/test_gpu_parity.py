@@ -1,0 +1,184 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle.
+
+Tolerances (fixed for the branch-decode step): attention output max abs error
+<= 1e-2 (bf16 output, fp32 accumulation), LSE within 1e-3, -inf LSE exactly
+where the oracle has no visible key; accepted lengths and tokens bit-exact.
+Small workloads are compared element by element; the full-size presets are
+compared on every row of a sample of branches chosen to include the extreme
+suffix lengths and every page boundary kind.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2607_18839_gb300 import workloads as W
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+OUT_TOL = 1e-2
+LSE_TOL = 1e-3
+
+
+@pytest.fixture(scope="module")
+def hpd():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2607_18839_gb300 import build, hpd as H
+    build.build()
+    H.load()
+    return H
+
+
+def run_gpu(H, inp):
+    d = H.DeviceInputs.from_host(inp)
+    op = H.BranchAttn(d)
+    out, lse = op()
+    torch.cuda.synchronize()
+    err = op.errors()
+    return out.float().cpu().numpy(), lse.cpu().numpy(), err
+
+
+def compare(inp, out, lse, ref_out, ref_lse, rows=None):
+    if rows is not None:
+        out, lse, ref_out, ref_lse = out[rows], lse[rows], ref_out[rows], ref_lse[rows]
+    neg = np.isneginf(ref_lse)
+    assert np.array_equal(np.isneginf(lse), neg), "-inf LSE pattern differs"
+    assert np.all(np.isfinite(lse[~neg]))
+    if (~neg).any():
+        lerr = np.max(np.abs(lse[~neg] - ref_lse[~neg]))
+        assert lerr <= LSE_TOL, f"lse err {lerr}"
+    oerr = np.max(np.abs(out - ref_out))
+    assert oerr <= OUT_TOL, f"out err {oerr}"
+    return oerr
+
+
+def branch_rows(inp, branches):
+    branches = np.asarray(branches)
+    return (branches[:, None] * inp.m + np.arange(inp.m)[None, :]).reshape(-1)
+
+
+SMALL = {
+    "c1": lambda: W.make_config("c1"),
+    "c2": lambda: W.make_config("c2"),
+    # several pages, ragged row tiles, private lengths 0 / < m / page multiples
+    "multi_page_ragged": lambda: W.build_inputs(
+        [300, 0, 77, 129], [3, 2, 1, 5], [0, 5, 16, 1, 40, 2, 31, 32, 48, 200, 3],
+        4, 16, 2, 128, seed=31, extra_pages=7),
+    "fork_prefix_lengths": lambda: W.build_inputs(
+        [500, 200], [4, 3], [10, 20, 30, 40, 0, 1, 2], 3, 8, 4, 128, seed=32,
+        branch_prefix_len=[500, 0, 1, 250, 200, 63, 64]),
+    "d64_g1": lambda: W.build_inputs([333], [5], [1, 17, 33, 65, 129], 2, 4, 4, 64, seed=33),
+    "g16_m16": lambda: W.build_inputs([100, 260], [2, 2], [0, 15, 16, 300], 16, 16, 1, 128,
+                                      seed=34),
+    "m1_empty_suffix": lambda: W.build_inputs([1152], [16], [0] * 16, 1, 16, 2, 128, seed=35),
+    "no_prefix_at_all": lambda: W.build_inputs([0], [3], [0, 4, 50], 4, 8, 2, 128, seed=36),
+    "long_suffix_splits": lambda: W.build_inputs([64], [2], [2047, 1500], 4, 32, 8, 128, seed=37,
+                                                 max_pages=129),
+    "custom_scale": lambda: W.build_inputs([90], [2], [7, 9], 2, 4, 2, 64, seed=38, scale=0.3),
+}
+
+
+@pytest.mark.parametrize("name", list(SMALL))
+def test_parity_small_elementwise(hpd, name):
+    inp = SMALL[name]()
+    ref_out, ref_lse = oracle.branch_attn(inp)
+    out, lse, err = run_gpu(hpd, inp)
+    assert err == 0
+    compare(inp, out, lse, ref_out, ref_lse)
+
+
+def sample_branches(inp, k=6):
+    s = inp.branch_len
+    picks = {0, inp.B - 1, int(np.argmax(s)), int(np.argmin(s))}
+    for d in (0, inp.n_docs - 1):
+        picks.update({int(inp.branch_cu[d]), int(inp.branch_cu[d + 1]) - 1})
+    rng = np.random.default_rng(5)
+    picks.update(rng.choice(inp.B, size=min(k, inp.B), replace=False).tolist())
+    return sorted(b for b in picks if 0 <= b < inp.B)
+
+
+@pytest.mark.parametrize("name", ["c3", "c4", "c5"])
+def test_parity_full_size_sampled_branches(hpd, name):
+    inp = W.make_config(name)
+    sel = np.array(sample_branches(inp), dtype=np.int32)
+    ref_out, ref_lse = oracle.branch_attn(inp, branch_sel=sel)
+    out, lse, err = run_gpu(hpd, inp)
+    assert err == 0
+    compare(inp, out, lse, ref_out, ref_lse, rows=branch_rows(inp, sel))
+    # every row is finite and every output is a convex combination of values
+    assert np.all(np.isfinite(lse)) and np.all(np.abs(out) <= 4.0)
+
+
+def test_c3_full_oracle_elementwise(hpd):
+    inp = W.make_config("c3")
+    ref_out, ref_lse = oracle.branch_attn(inp)
+    out, lse, _ = run_gpu(hpd, inp)
+    compare(inp, out, lse, ref_out, ref_lse)
+
+
+def test_repeated_calls_are_deterministic(hpd):
+    inp = W.make_config("c2")
+    d = hpd.DeviceInputs.from_host(inp)
+    op = hpd.BranchAttn(d)
+    o1 = op()[0].clone()
+    o2 = op()[0].clone()
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2)
+
+
+def test_out_of_range_device_data_is_clamped_and_flagged(hpd):
+    inp = W.build_inputs([40], [2], [20, 30], 2, 8, 2, 64, seed=39)
+    inp.page_table[1, 0] = inp.num_pages + 5   # page id out of range
+    inp.branch_len[0] = 10_000                   # beyond the page table
+    out, lse, err = run_gpu(hpd, inp)
+    assert err & 0x8 and err & 0x4
+    assert np.all(np.isfinite(out))
+
+
+# ------------------------------------------------------------- acceptance --
+
+def run_accept(hpd, logits_bits, drafts):
+    lg = torch.from_numpy(np.ascontiguousarray(logits_bits).view(np.int16)).cuda().view(torch.bfloat16)
+    dr = torch.from_numpy(np.ascontiguousarray(drafts, dtype=np.int32)).cuda()
+    tok, acc = hpd.pmtp_accept(lg, dr)
+    torch.cuda.synchronize()
+    return tok.cpu().numpy(), acc.cpu().numpy()
+
+
+def test_accept_c5_bit_exact(hpd):
+    logits = W.accept_inputs()
+    ref_tok0, _ = oracle.pmtp_accept(logits, np.zeros(logits.shape[:2], np.int32))
+    drafts = W.mix_drafts(ref_tok0, logits.shape[2], 0.7, seed=77)
+    ref_tok, ref_acc = oracle.pmtp_accept(logits, drafts)
+    tok, acc = run_accept(hpd, logits, drafts)
+    np.testing.assert_array_equal(tok, ref_tok)
+    np.testing.assert_array_equal(acc, ref_acc)
+    assert 0 < ref_acc.mean() < 4
+
+
+@pytest.mark.parametrize("V", [1, 7, 8, 9, 4095, 32001])
+def test_accept_ragged_vocab_ties_and_nan(hpd, V):
+    rng = np.random.default_rng(V)
+    B, m = 5, 6
+    vals = rng.integers(-3, 4, size=(B, m, V)).astype(np.float32)  # many ties
+    vals[0, 0, :] = np.nan
+    vals[1, 1, V // 2] = np.nan
+    vals[2, 2, :] = -np.inf
+    logits = W.f32_to_bf16_bits(vals)
+    ref_tok0, _ = oracle.pmtp_accept(logits, np.zeros((B, m), np.int32))
+    drafts = W.mix_drafts(ref_tok0, V, 0.8, seed=V + 1)
+    ref_tok, ref_acc = oracle.pmtp_accept(logits, drafts)
+    tok, acc = run_accept(hpd, logits, drafts)
+    np.testing.assert_array_equal(tok, ref_tok)
+    np.testing.assert_array_equal(acc, ref_acc)
+
+
+def test_accept_misaligned_rows(hpd):
+    # V = 33 makes every row start at a different 16-byte phase
+    rng = np.random.default_rng(2)
+    logits = W.f32_to_bf16_bits(rng.standard_normal((9, 7, 33)).astype(np.float32))
+    ref_tok, ref_acc = oracle.pmtp_accept(logits, np.zeros((9, 7), np.int32))
+    tok, acc = run_accept(hpd, logits, np.zeros((9, 7), np.int32))
+    np.testing.assert_array_equal(tok, ref_tok)
+    np.testing.assert_array_equal(acc, ref_acc)
