@@ -155,6 +155,37 @@ hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *args, hpd_stream_t
 hpd_status hpd_pmtp_accept(const void *logits, const int32_t *drafts, int B, int m, int V,
                            int32_t *out_tokens, int32_t *accepted_len, hpd_stream_t stream);
 
+/*
+ * hpd_branch_attn for callers that cannot allocate device memory.  The
+ * paper has no counterpart to this entry point.
+ *
+ * Some callers of this library cannot obtain a workspace: a plugin whose
+ * host engine owns all device memory and passes it only its inputs and
+ * outputs, or code on a path where cudaMalloc (which can synchronise the
+ * whole device) is not allowed.  This variant computes exactly what
+ * hpd_branch_attn computes, but keeps its scratch in a file-scope device
+ * array of HPD_NOALLOC_WORKSPACE_BYTES inside libhpd, which every GPU that
+ * loads the library holds until the process exits.  args->workspace and
+ * args->workspace_bytes are ignored (they may be NULL / 0); every other
+ * field means what it means for hpd_branch_attn.
+ *   - Nothing is allocated: no cudaMalloc, cudaFree or allocating library
+ *     routine is called.
+ *   - A shape whose hpd_branch_attn_workspace_size exceeds
+ *     HPD_NOALLOC_WORKSPACE_BYTES is rejected with HPD_ERR_WORKSPACE before
+ *     anything is enqueued.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current); make that first call
+ *     before any stream capture on the device.
+ *   - All calls share the one array, which keeps the previous call's
+ *     contents; each call clears its error word on `stream` first.  Calls
+ *     whose work overlaps on the GPU (other streams, other threads) race on
+ *     the array and give undefined results: serialise them.
+ *   - The clamp flags of the device-side checks are kept in the shared array
+ *     and are not reported (hpd_read_errors needs a caller workspace).
+ */
+#define HPD_NOALLOC_WORKSPACE_BYTES (32u << 20)
+hpd_status hpd_branch_attn_noalloc(const hpd_branch_attn_args *args, hpd_stream_t stream);
+
 /* Copy the workspace error word (HPD_DEVERR_* bits) to *flags.  This is the
  * one call that synchronises: it waits for `stream`. */
 hpd_status hpd_read_errors(const void *workspace, uint32_t *flags, hpd_stream_t stream);

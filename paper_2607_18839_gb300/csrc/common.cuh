@@ -123,6 +123,8 @@ namespace hpd {
 cudaError_t launch_prefix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
 cudaError_t launch_suffix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
 cudaError_t launch_merge(const MergeParams &p, cudaStream_t s);
+// Remember `e` for hpd_last_cuda_error() and return HPD_ERR_CUDA.
+hpd_status record_cuda_error(cudaError_t e);
 cudaError_t launch_accept(const __nv_bfloat16 *logits, const int32_t *drafts, int B, int m, int V,
                           int32_t *out_tokens, int32_t *accepted_len, cudaStream_t s);
 }  // namespace hpd

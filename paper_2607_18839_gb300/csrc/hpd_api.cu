@@ -74,6 +74,8 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
 
 }  // namespace
 
+hpd_status hpd::record_cuda_error(cudaError_t e) { return cuda_fail(e); }
+
 extern "C" {
 
 size_t hpd_branch_attn_workspace_size(const hpd_branch_attn_args *args) {

@@ -25,7 +25,10 @@ DEVERR = {0x1: "PREFIX_CU", 0x2: "BRANCH_CU", 0x4: "BRANCH_LEN", 0x8: "PAGE_ID",
 # Every entry point declared in include/hpd.h.
 EXPORTS = ("hpd_branch_attn_workspace_size", "hpd_workspace_init", "hpd_branch_attn",
            "hpd_branch_attn_launches", "hpd_branch_attn_marked", "hpd_pmtp_accept", "hpd_read_errors", "hpd_status_string", "hpd_last_cuda_error",
-           "hpd_version")
+           "hpd_version", "hpd_branch_attn_noalloc")
+
+# Scratch bytes built into libhpd for hpd_branch_attn_noalloc.
+NOALLOC_WORKSPACE_BYTES = 32 << 20
 
 
 class HpdError(RuntimeError):
@@ -87,6 +90,8 @@ def load(path: str = LIB_PATH):
     lib.hpd_last_cuda_error.argtypes = []
     lib.hpd_version.restype = I
     lib.hpd_version.argtypes = []
+    lib.hpd_branch_attn_noalloc.restype = I
+    lib.hpd_branch_attn_noalloc.argtypes = [ctypes.POINTER(hpd_branch_attn_args), P]
     _lib = lib
     return lib
 
@@ -147,6 +152,13 @@ def hpd_read_errors(workspace_ptr: int, stream_handle) -> int:
     _check("hpd_read_errors", load().hpd_read_errors(workspace_ptr, ctypes.byref(flags),
                                                       stream_handle))
     return int(flags.value)
+
+
+def hpd_branch_attn_noalloc(args: hpd_branch_attn_args, stream_handle: Optional[int]) -> None:
+    """The step with libhpd's built-in scratch array instead of a workspace
+    (for callers that cannot allocate; see include/hpd.h)."""
+    _check("hpd_branch_attn_noalloc", load().hpd_branch_attn_noalloc(ctypes.byref(args),
+                                                                      stream_handle))
 
 
 def hpd_status_string(status: int) -> str:
