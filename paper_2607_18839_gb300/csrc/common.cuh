@@ -24,6 +24,7 @@ struct Plan {
   int tiles_max;   // upper bound of prefix row tiles per KV head
   int wr_s;        // warps along rows in the suffix kernel (1, 2, 4)
   int rt_s;        // suffix row tiles per (branch, KV head)
+  bool use_tc;     // prefix stage on tcgen05 (G divides 128) or warp MMA
   size_t off_err;    // uint32 error word
   size_t off_opart;  // fp32 [S_p + S_s][rows_total][H_q][D]
   size_t off_lpart;  // fp32 [S_p + S_s][rows_total][H_q]
@@ -121,6 +122,7 @@ __device__ __forceinline__ int ceil_div_i(int a, int b) { return (a + b - 1) / b
 // Host-side launchers (defined in the .cu files, called by hpd_api.cu).
 namespace hpd {
 cudaError_t launch_prefix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
+cudaError_t launch_prefix_stage_tc(const AttnParams &p, const Plan &plan, cudaStream_t s);
 cudaError_t launch_suffix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
 cudaError_t launch_merge(const MergeParams &p, cudaStream_t s);
 // Remember `e` for hpd_last_cuda_error() and return HPD_ERR_CUDA.

@@ -18,7 +18,9 @@ hpd_status cuda_fail(cudaError_t e) {
 
 constexpr size_t kAlign = 256;
 constexpr int kPrefixTileRows = 64;   // rows per prefix-stage CTA
-constexpr int kTargetCtas = 152 * 4;  // prefix-stage CTAs aimed for (GB300: 152 SMs)
+constexpr int kPlanSms = 148;          // SMs the split plan assumes (GB300)
+constexpr int kTargetCtas = kPlanSms * 4;  // warp-MMA prefix CTAs aimed for
+constexpr int kTcTileRows = 128;       // stacked rows of one tcgen05 prefix CTA
 constexpr int kMaxPrefixSplits = 16;
 constexpr int kSuffixSplitKeys = 1024;  // a suffix chunk holds at most ~this many keys
 constexpr int kMaxSuffixSplits = 8;
@@ -49,15 +51,26 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
   hpd::Plan pl{};
   pl.G = a->H_q / a->H_kv;
   pl.rows_total = a->B * a->m;
-  const long long stacked = static_cast<long long>(a->B) * a->m * pl.G;
-  const int tiles = ceil_div(stacked, kPrefixTileRows);
-  pl.tiles_max = tiles + a->n_docs;
   const int maxP = a->max_prefix_len > 0 ? std::min(a->max_prefix_len, a->prefix_tokens)
                                          : a->prefix_tokens;
-  const long long tiles_est = static_cast<long long>(std::max(tiles, 1)) * a->H_kv;
-  int sp = ceil_div(kTargetCtas, tiles_est);
-  sp = std::min(sp, std::max(1, ceil_div(maxP, 256)));
-  pl.S_p = std::max(1, std::min(sp, kMaxPrefixSplits));
+  pl.use_tc = (a->D == 64 || a->D == 128) && (kTcTileRows % pl.G == 0);
+  if (pl.use_tc) {
+    // tcgen05 stage: 128 stacked rows (128 / G tokens) per CTA, one CTA per SM
+    const int tiles = ceil_div(static_cast<long long>(a->B) * a->m, kTcTileRows / pl.G);
+    pl.tiles_max = tiles + a->n_docs;
+    const long long tiles_est = static_cast<long long>(std::max(tiles, 1)) * a->H_kv;
+    int sp = ceil_div(2LL * kPlanSms, tiles_est);
+    sp = std::min(sp, std::max(1, maxP / 256));
+    pl.S_p = std::max(1, std::min(sp, kMaxPrefixSplits));
+  } else {
+    const long long stacked = static_cast<long long>(a->B) * a->m * pl.G;
+    const int tiles = ceil_div(stacked, kPrefixTileRows);
+    pl.tiles_max = tiles + a->n_docs;
+    const long long tiles_est = static_cast<long long>(std::max(tiles, 1)) * a->H_kv;
+    int sp = ceil_div(kTargetCtas, tiles_est);
+    sp = std::min(sp, std::max(1, ceil_div(maxP, 256)));
+    pl.S_p = std::max(1, std::min(sp, kMaxPrefixSplits));
+  }
   const int maxL = a->max_pages_per_branch * hpd::kPage;
   pl.S_s = std::max(1, std::min(ceil_div(maxL, kSuffixSplitKeys), kMaxSuffixSplits));
   const int rows_s = a->m * pl.G;
@@ -153,7 +166,8 @@ hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t st
     return cudaEventRecordWithFlags(static_cast<cudaEvent_t>(ev[k]), s, cudaEventRecordExternal);
   };
   cudaError_t e = mark(0);
-  if (e == cudaSuccess) e = hpd::launch_prefix_stage(p, pl, s);
+  if (e == cudaSuccess)
+    e = pl.use_tc ? hpd::launch_prefix_stage_tc(p, pl, s) : hpd::launch_prefix_stage(p, pl, s);
   if (e == cudaSuccess) e = mark(1);
   if (e == cudaSuccess) e = hpd::launch_suffix_stage(p, pl, s);
   if (e == cudaSuccess) e = mark(2);

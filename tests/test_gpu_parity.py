@@ -76,6 +76,15 @@ SMALL = {
     "long_suffix_splits": lambda: W.build_inputs([64], [2], [2047, 1500], 4, 32, 8, 128, seed=37,
                                                  max_pages=129),
     "custom_scale": lambda: W.build_inputs([90], [2], [7, 9], 2, 4, 2, 64, seed=38, scale=0.3),
+    # G = 3 and G = 5 do not divide 128: these take the warp-MMA prefix kernel
+    "g3_warp_mma_prefix": lambda: W.build_inputs([200, 50], [3, 2], [4, 0, 33, 17, 64], 3, 6, 2,
+                                                 128, seed=42, branch_prefix_len=[200, 7, 150, 50, 0]),
+    "g5_d64_warp_mma_prefix": lambda: W.build_inputs([129], [4], [1, 2, 3, 100], 2, 10, 2, 64,
+                                                     seed=43),
+    # many pages with one branch each, long prefixes split across CTAs
+    "many_pages_split_prefix": lambda: W.build_inputs([1000 + 37 * i for i in range(12)], [1] * 12,
+                                                      [5 * i for i in range(12)], 4, 16, 2, 128,
+                                                      seed=44),
 }
 
 
