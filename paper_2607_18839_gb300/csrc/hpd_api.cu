@@ -18,10 +18,10 @@ hpd_status cuda_fail(cudaError_t e) {
 
 constexpr size_t kAlign = 256;
 constexpr int kPrefixTileRows = 64;   // rows per prefix-stage CTA
-constexpr int kPlanSms = 148;          // SMs the split plan assumes (GB300)
+constexpr int kPlanSms = 152;          // SMs the split plan assumes (GB300)
 constexpr int kTargetCtas = kPlanSms * 4;  // warp-MMA prefix CTAs aimed for
 constexpr int kTcTileRows = 128;       // stacked rows of one tcgen05 prefix CTA
-constexpr int kMaxPrefixSplits = 16;
+constexpr int kMaxPrefixSplits = 8;
 constexpr int kSuffixSplitKeys = 1024;  // a suffix chunk holds at most ~this many keys
 constexpr int kMaxSuffixSplits = 8;
 
@@ -55,13 +55,29 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
                                          : a->prefix_tokens;
   pl.use_tc = (a->D == 64 || a->D == 128) && (kTcTileRows % pl.G == 0);
   if (pl.use_tc) {
-    // tcgen05 stage: 128 stacked rows (128 / G tokens) per CTA, one CTA per SM
-    const int tiles = ceil_div(static_cast<long long>(a->B) * a->m, kTcTileRows / pl.G);
+    // tcgen05 stage: NT tiles of 128 stacked rows (128 / G tokens each) per
+    // CTA, one CTA per SM.  Two tiles share every K / V load when pages are
+    // big enough to fill them.
+    const long long stacked = static_cast<long long>(a->B) * a->m * pl.G;
+    pl.tc_tiles = stacked >= 2LL * kTcTileRows * a->n_docs ? 2 : 1;
+    const int tile_tokens = pl.tc_tiles * (kTcTileRows / pl.G);
+    const int tiles = ceil_div(static_cast<long long>(a->B) * a->m, tile_tokens);
     pl.tiles_max = tiles + a->n_docs;
-    const long long tiles_est = static_cast<long long>(std::max(tiles, 1)) * a->H_kv;
-    int sp = ceil_div(2LL * kPlanSms, tiles_est);
-    sp = std::min(sp, std::max(1, maxP / 256));
-    pl.S_p = std::max(1, std::min(sp, kMaxPrefixSplits));
+    // Key splits: the fewest waves of CTAs x blocks per CTA (+2 blocks of
+    // prologue / epilogue per CTA), for the longest page.
+    const long long ctas = static_cast<long long>(std::max(tiles, 1)) * a->H_kv;
+    const int nb = std::max(1, ceil_div(maxP, 128));
+    int best = 1;
+    long long best_cost = -1;
+    for (int sp = 1; sp <= std::min(nb, kMaxPrefixSplits); ++sp) {
+      const long long waves = (ctas * sp + kPlanSms - 1) / kPlanSms;
+      const long long cost = waves * (ceil_div(nb, sp) + 2);
+      if (best_cost < 0 || cost < best_cost) {
+        best_cost = cost;
+        best = sp;
+      }
+    }
+    pl.S_p = best;
   } else {
     const long long stacked = static_cast<long long>(a->B) * a->m * pl.G;
     const int tiles = ceil_div(stacked, kPrefixTileRows);
