@@ -2,8 +2,9 @@
 """Benchmark of the branch-decode step of Hierarchical Parallel Decoding.
 
 One step = one pass of the whole hot path over one batch of synthetic input:
-hpd_branch_attn (shared-prefix stage, private-suffix stage, LSE merge over the
-paged KV) followed by hpd_pmtp_accept (greedy verification of the P-MTP
+hpd_branch_attn (the tcgen05 shared-prefix stage, then the private-suffix
+stage over the paged KV, which also does the LSE merge) followed by
+hpd_pmtp_accept (greedy verification of the P-MTP
 drafts against bf16 logits over a 32,000-token vocabulary).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c2]
@@ -47,7 +48,7 @@ METRIC = "branch-decode query-tokens/s"
 UNIT = "query-tokens/s"
 VOCAB = 32000
 DRAFT_MATCH = 0.7
-KERNELS = ("prefix_stage", "suffix_stage", "lse_merge", "pmtp_accept")
+ACCEPT = "pmtp_accept"
 
 
 # ------------------------------------------------------------------ helpers --
@@ -84,10 +85,14 @@ def algorithmic_work(inp, V=VOCAB):
     suffix_flops = 4.0 * Hq * D * vis.sum()
     accept_bytes = rows * V * 2 + rows * 4 * 2 + inp.B * 4
     per = {
+        # tcgen05 path: one kernel for prefix + suffix (+ merge of key splits)
+        "branch_attn_tc": dict(bytes=prefix_kv + private_kv + q_bytes + tables + out_bytes,
+                               flops=prefix_flops + suffix_flops),
+        "merge_splits": dict(bytes=out_bytes, flops=0.0),
+        # warp-MMA path (G not dividing 128)
         "prefix_stage": dict(bytes=prefix_kv + q_bytes, flops=prefix_flops),
-        "suffix_stage": dict(bytes=private_kv + q_bytes + tables, flops=suffix_flops),
-        "lse_merge": dict(bytes=out_bytes, flops=0.0),
-        "pmtp_accept": dict(bytes=accept_bytes, flops=0.0),
+        "suffix_merge": dict(bytes=private_kv + q_bytes + tables + out_bytes, flops=suffix_flops),
+        ACCEPT: dict(bytes=accept_bytes, flops=0.0),
     }
     step_bytes = q_bytes + prefix_kv + private_kv + tables + out_bytes + accept_bytes
     return per, dict(bytes=step_bytes, flops=prefix_flops + suffix_flops)
@@ -176,7 +181,7 @@ def oracle_sample_run(inp, logits, drafts, budget_s: float, rng_seed: int = 0):
     sample description)."""
     import oracle
     per, _ = algorithmic_work(inp)
-    est_flops = 2.0 * (per["prefix_stage"]["flops"] + per["suffix_stage"]["flops"]) / inp.B
+    est_flops = 2.0 * (per["branch_attn_tc"]["flops"]) / inp.B
     threads = oracle.max_threads()
     per_branch_s = est_flops / (0.5e9 * threads)  # ~0.5 GFLOP/s per thread, fp64 scalar loops
     n = int(max(1, min(inp.B, budget_s / 3.0 / max(per_branch_s, 1e-9))))
@@ -237,6 +242,7 @@ def run_ours(args, world, rank, local):
         return H.DeviceInputs(**{k: (v.clone() if isinstance(v, torch.Tensor) else v)
                                  for k, v in d.__dict__.items()})
 
+    # (the library keeps raw device pointers: these lists keep the tensors alive)
     reps = [base] + [clone_inputs(base) for _ in range(R - 1)]
     logits = [logits0] + [logits0.clone() for _ in range(R - 1)]
     op = H.BranchAttn(base, stream=stream)
@@ -255,13 +261,19 @@ def run_ours(args, world, rank, local):
     drafts_np = W.mix_drafts(out_tokens.cpu().numpy(), VOCAB, DRAFT_MATCH, seed=3000 + rank)
     drafts = torch.from_numpy(drafts_np).to(dev)
 
-    def step(r, ev=None):
+    def attn(r, ev=None):
         if ev is None:
             H.hpd_branch_attn(argsets[r], sh)
         else:
             H.hpd_branch_attn_marked(argsets[r], sh, ev)
+
+    def accept(r):
         H.hpd_pmtp_accept(logits[r].data_ptr(), drafts.data_ptr(), inp.B, inp.m, VOCAB,
                           out_tokens.data_ptr(), acc.data_ptr(), sh)
+
+    def step(r, ev=None):
+        attn(r, ev)
+        accept(r)
 
     # ---- warm-up (eager), also sets the kernels' function attributes
     with torch.cuda.stream(stream):
@@ -272,48 +284,42 @@ def run_ours(args, world, rank, local):
     if err:
         raise SystemExit(f"bench.py: device error flags {err:#x}")
 
-    # ---- graphs of S steps, each step with timing markers
+    # ---- CUDA graphs of S steps (inputs rotated over the R replicas)
     K = args.steps
     S = max(1, min(K, args.graph_steps))
-    events = [[torch.cuda.Event(enable_timing=True) for _ in range(n_launch + 1)] for _ in range(S)]
-    with torch.cuda.stream(stream):
-        for row in events:
-            for e in row:
-                e.record(stream)  # creates the handle
-    stream.synchronize()
-    handles = [[int(e.cuda_event) for e in row] for row in events]
 
-    def capture(nsteps, offset, with_events, h2d=None, d2h=None):
+    def capture(nsteps, offset, body):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
             for i in range(nsteps):
-                r = (offset + i) % R
-                if h2d is not None:
-                    h2d(r)
-                step(r, handles[i] if with_events else None)
-                if d2h is not None:
-                    d2h()
+                body((offset + i) % R, i)
         return g
 
-    g_main = capture(S, 0, True)
-    g_rem = capture(K % S, S, False) if K % S else None
+    g_main = capture(S, 0, lambda r, i: step(r))
+    g_rem = capture(K % S, S, lambda r, i: step(r)) if K % S else None
     n_main = K // S
 
-    def timed(gm, gr, nm):
-        if world > 1:
+    wall_ms = [0.0]  # host wall clock of the last timed region (cross-check)
+
+    def timed(gm, gr, nm, sync_ranks=True):
+        if world > 1 and sync_ranks:
             dist.barrier()
         torch.cuda.synchronize(dev)
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
-        t0.record(stream)
-        for _ in range(nm):
-            gm.replay()
-        if gr is not None:
-            gr.replay()
-        t1.record(stream)
+        w0 = time.perf_counter()
+        # replay() launches on the current stream: make it the timing stream
+        with torch.cuda.stream(stream):
+            t0.record(stream)
+            for _ in range(nm):
+                gm.replay()
+            if gr is not None:
+                gr.replay()
+            t1.record(stream)
         torch.cuda.synchronize(dev)
+        wall_ms[0] = (time.perf_counter() - w0) * 1e3
         ms = t0.elapsed_time(t1)
-        if world > 1:
+        if world > 1 and sync_ranks:
             t = torch.tensor([ms], dtype=torch.float64, device=dev)
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
             dist.barrier()
@@ -325,19 +331,34 @@ def run_ours(args, world, rank, local):
     clocks = ClockSampler(gpu_id)
     clocks.start()
     total_ms = timed(g_main, g_rem, n_main)
+    total_wall_ms = wall_ms[0]
     clk = clocks.stop()
 
-    # per-kernel durations: markers of the last replay of the S-step graph
-    # (steps i and i+1 bracket step i's acceptance kernel)
-    per_kernel = {k: [] for k in KERNELS}
-    for i in range(S):
-        ev = events[i]
-        per_kernel["prefix_stage"].append(ev[0].elapsed_time(ev[1]))
-        per_kernel["suffix_stage"].append(ev[1].elapsed_time(ev[2]))
-        per_kernel["lse_merge"].append(ev[2].elapsed_time(ev[3]))
-        if i + 1 < S:
-            per_kernel["pmtp_accept"].append(ev[n_launch].elapsed_time(events[i + 1][0]))
-    kernel_ms = {k: (statistics.mean(v) if v else None) for k, v in per_kernel.items()}
+    # ---- per-kernel durations, measured right after the timed region on the
+    # same stream: the attention call and the acceptance kernel each replayed
+    # back to back from their own graphs (events around the replays), and the
+    # attention call's kernels apportioned by timing markers recorded inside a
+    # graph of marked calls.
+    n_rep = max(1, (2 * K) // S)
+    g_attn = capture(S, 0, lambda r, i: attn(r))
+    g_acc = capture(S, 0, lambda r, i: accept(r))
+    attn_ms = timed(g_attn, None, n_rep, sync_ranks=False) / (n_rep * S)
+    acc_ms = timed(g_acc, None, n_rep, sync_ranks=False) / (n_rep * S)
+    attn_names = [H.hpd_branch_attn_kernel_name(argsets[0], k) for k in range(n_launch)]
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(n_launch + 1)] for _ in range(S)]
+    with torch.cuda.stream(stream):
+        for row in events:
+            for e in row:
+                e.record(stream)  # creates the handle
+    stream.synchronize()
+    handles = [[int(e.cuda_event) for e in row] for row in events]
+    g_mark = capture(S, 0, lambda r, i: attn(r, handles[i]))
+    with torch.cuda.stream(stream):
+        g_mark.replay()
+    torch.cuda.synchronize(dev)
+    span = [statistics.mean(ev[k].elapsed_time(ev[k + 1]) for ev in events) for k in range(n_launch)]
+    kernel_ms = {name: attn_ms * span[k] / sum(span) for k, name in enumerate(attn_names)}
+    kernel_ms[ACCEPT] = acc_ms
 
     # ---- end to end: pinned host inputs in, results out, every step
     host_q = torch.from_numpy(inp.q.view(np.int16)).pin_memory()
@@ -367,8 +388,13 @@ def run_ours(args, world, rank, local):
     h2d_bytes = sum(t.numel() * t.element_size()
                     for t in [host_q, *host_meta, host_logits, host_drafts])
     d2h_bytes = sum(t.numel() * t.element_size() for t in (host_out, host_lse, host_tok, host_acc))
-    ge_main = capture(S, 0, False, h2d, d2h)
-    ge_rem = capture(K % S, S, False, h2d, d2h) if K % S else None
+    def e2e_step(r, i):
+        h2d(r)
+        step(r)
+        d2h()
+
+    ge_main = capture(S, 0, e2e_step)
+    ge_rem = capture(K % S, S, e2e_step) if K % S else None
     e2e_ms = timed(ge_main, ge_rem, n_main)
     err = op.errors(stream)
     if err:
@@ -395,7 +421,9 @@ def run_ours(args, world, rank, local):
     known = {k: v for k, v in kernel_ms.items() if v is not None}
     dom = max(known, key=known.get)
     dom_ms = known[dom]
-    if per[dom]["flops"] > 0 and dom == "prefix_stage":
+    t_bytes = per[dom]["bytes"] / (pk["hbm"] * 1e9)
+    t_flops = per[dom]["flops"] / (pk["tc_sustained"] * 1e12)
+    if t_flops > t_bytes:
         achieved = per[dom]["flops"] / (dom_ms * 1e-3) / 1e12
         roof = {"bound": "tensor", "achieved": achieved, "peak": pk["tc_sustained"],
                 "unit": "TFLOP/s"}
@@ -418,7 +446,8 @@ def run_ours(args, world, rank, local):
             "query_tokens_per_step": qtok,
             "l2": f"{R} rotating input replicas ({R * rep_bytes / 2**20:.0f} MiB > 3x L2 "
                   f"{l2 / 2**20:.0f} MiB)",
-            "timing": f"CUDA graphs of {S} steps, events on the launch stream",
+            "timing": f"CUDA graphs of {S} steps, events on the launch stream; per-kernel "
+                      f"times from back-to-back graphs of each call after the timed region",
             "parallelism": f"dp{world} (independent pages per GPU, no collective)",
         },
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
@@ -431,7 +460,9 @@ def run_ours(args, world, rank, local):
         "step_roofline": {"bytes": step_work["bytes"], "flops": step_work["flops"],
                           "t_roofline_us": t_roof * 1e6,
                           "frac": t_roof / (ms_step * 1e-3)},
-        "kernel_us": {k: (v * 1e3 if v is not None else None) for k, v in kernel_ms.items()},
+        "kernel_us": {k: v * 1e3 for k, v in kernel_ms.items()},
+        "attn_call_us": attn_ms * 1e3,
+        "host_wall_ms_per_step": total_wall_ms / K,
         "cpu_baseline": cpu,
         "clocks": clk,
     }
@@ -453,7 +484,7 @@ def run_reference(args, world, rank):
     drafts = W.mix_drafts(tok, VOCAB, DRAFT_MATCH, seed=3000)
     per, _ = algorithmic_work(inp)
     threads = oracle.max_threads()
-    est = 2.0 * (per["prefix_stage"]["flops"] + per["suffix_stage"]["flops"]) / inp.B
+    est = 2.0 * (per["branch_attn_tc"]["flops"]) / inp.B
     n = int(max(1, min(inp.B, args.ref_step_seconds / max(est / (0.5e9 * threads), 1e-9))))
     rng = np.random.default_rng(0)
     sel = np.sort(rng.choice(inp.B, size=n, replace=False)).astype(np.int32)

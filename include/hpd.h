@@ -116,8 +116,9 @@ typedef struct {
  * invalid. */
 size_t hpd_branch_attn_workspace_size(const hpd_branch_attn_args *args);
 
-/* Zero the workspace (error word and internal counters) on `stream`.  Call
- * once after allocating it; hpd_branch_attn leaves it reusable. */
+/* Zero the workspace (error word and arrival tickets) on `stream`.  Call
+ * once after allocating it; every hpd_branch_attn call leaves the tickets
+ * at zero again, so the workspace stays reusable. */
 hpd_status hpd_workspace_init(void *workspace, size_t workspace_bytes, hpd_stream_t stream);
 
 /* The branch-decode attention step (see the struct above).  Enqueues its
@@ -126,9 +127,15 @@ hpd_status hpd_workspace_init(void *workspace, size_t workspace_bytes, hpd_strea
 hpd_status hpd_branch_attn(const hpd_branch_attn_args *args, hpd_stream_t stream);
 
 /* Number of kernels one hpd_branch_attn call launches for these scalars
- * (0 if they are invalid): the shared-prefix stage, the private-suffix stage
- * and the log-sum-exp merge, in that order. */
+ * (0 if they are invalid).  When H_q / H_kv divides 128 the step runs on
+ * tcgen05 tensor cores: one kernel for the shared prefix and the private
+ * suffixes, plus a merge kernel when the keys are split across CTAs.
+ * Otherwise: a warp-MMA shared-prefix kernel, then a warp-MMA private-suffix
+ * kernel that also merges and writes out / lse. */
 int hpd_branch_attn_launches(const hpd_branch_attn_args *args);
+
+/* Name of the k-th of those kernels (static string), or NULL. */
+const char *hpd_branch_attn_kernel_name(const hpd_branch_attn_args *args, int k);
 
 /* hpd_branch_attn with timing markers.  stage_events holds
  * hpd_branch_attn_launches(args) + 1 cudaEvent_t handles created by the

@@ -1,69 +1,10 @@
-// merge_accept.cu -- the log-sum-exp merge of the split partials and the
-// greedy P-MTP acceptance kernel.
+// accept.cu -- the greedy P-MTP acceptance kernel.
 #include <climits>
 
 #include "common.cuh"
 
 namespace hpd {
 namespace {
-
-// One warp per (query token, query head): combine the S_total partials
-//   O = sum_s e^{lse_s - M} O_s / sum_s e^{lse_s - M},
-//   lse = M + ln sum_s e^{lse_s - M},   M = max_s lse_s,
-// skipping partials whose chunk had no visible key (lse_s = -inf).  The union
-// of the chunks is exactly the branch's visible key set (Sec. 3.3), so the
-// result equals one softmax over all of it.
-template <int D>
-__global__ void __launch_bounds__(256) merge_kernel(const MergeParams p) {
-  constexpr int E = D / 32;  // values per lane
-  const int lane = threadIdx.x & 31;
-  const long long pair = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  const long long n_pairs = static_cast<long long>(p.rows_total) * p.H_q;
-  if (pair >= n_pairs) return;
-  const float NEG_INF = -__int_as_float(0x7f800000);
-
-  const float ls = lane < p.S_total ? p.l_part[lane * n_pairs + pair] : NEG_INF;
-  float M = ls;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-
-  float acc[E];
-#pragma unroll
-  for (int e = 0; e < E; ++e) acc[e] = 0.f;
-  float lse_out = NEG_INF;
-  if (M != NEG_INF) {
-    const float w_lane = ls == NEG_INF ? 0.f : exp2f((ls - M) * kLog2e);
-    float wsum = w_lane;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) wsum += __shfl_xor_sync(0xffffffffu, wsum, o);
-    for (int s = 0; s < p.S_total; ++s) {
-      const float w = __shfl_sync(0xffffffffu, w_lane, s);
-      if (w == 0.f) continue;
-      const float *src = p.o_part + (s * n_pairs + pair) * D + lane * E;
-      if constexpr (E == 4) {
-        const float4 v = *reinterpret_cast<const float4 *>(src);
-        acc[0] += w * v.x; acc[1] += w * v.y; acc[2] += w * v.z; acc[3] += w * v.w;
-      } else {
-        const float2 v = *reinterpret_cast<const float2 *>(src);
-        acc[0] += w * v.x; acc[1] += w * v.y;
-      }
-    }
-    const float inv = 1.f / wsum;
-#pragma unroll
-    for (int e = 0; e < E; ++e) acc[e] *= inv;
-    lse_out = M + logf(wsum);
-  }
-  __nv_bfloat16 *dst = p.out + pair * D + lane * E;
-  if constexpr (E == 4) {
-    uint2 w;
-    w.x = pack_bf16x2(acc[0], acc[1]);
-    w.y = pack_bf16x2(acc[2], acc[3]);
-    *reinterpret_cast<uint2 *>(dst) = w;
-  } else {
-    *reinterpret_cast<uint32_t *>(dst) = pack_bf16x2(acc[0], acc[1]);
-  }
-  if (p.lse && lane == 0) p.lse[pair] = lse_out;
-}
 
 // ------------------------------------------------------------ acceptance --
 constexpr int kAcceptThreads = 512;
@@ -169,17 +110,6 @@ __global__ void __launch_bounds__(kAcceptThreads)
 }
 
 }  // namespace
-
-cudaError_t launch_merge(const MergeParams &p, cudaStream_t s) {
-  const long long n_pairs = static_cast<long long>(p.rows_total) * p.H_q;
-  const long long blocks = (n_pairs * 32 + 255) / 256;
-  if (blocks <= 0) return cudaSuccess;
-  if (p.D == 64)
-    merge_kernel<64><<<static_cast<unsigned>(blocks), 256, 0, s>>>(p);
-  else
-    merge_kernel<128><<<static_cast<unsigned>(blocks), 256, 0, s>>>(p);
-  return cudaGetLastError();
-}
 
 cudaError_t launch_accept(const __nv_bfloat16 *logits, const int32_t *drafts, int B, int m, int V,
                           int32_t *out_tokens, int32_t *accepted_len, cudaStream_t s) {

@@ -25,6 +25,7 @@ namespace {
 
 constexpr int kThreads = 128;  // 4 warps
 constexpr int kBN = 64;        // keys per shared-memory block
+constexpr int kMaxSlots = 17;  // prefix splits + suffix splits + own partial
 
 // Byte offset of 16-byte chunk `c` of row `r` in a row-major tile of D bf16
 // columns; chunks are XOR-swizzled by the row so ldmatrix is conflict-free.
@@ -179,7 +180,8 @@ __global__ void __launch_bounds__(kThreads) attn_stage_kernel(const AttnParams p
   };
 
   if (nrows <= 0) return;
-  if (k_end <= k_begin) {
+  const bool empty = k_end <= k_begin;
+  if (PREFIX && empty) {
     for (int r = tid; r < nrows; r += kThreads) p.l_part[out_index(r)] = NEG_INF;
     return;
   }
@@ -210,7 +212,7 @@ __global__ void __launch_bounds__(kThreads) attn_stage_kernel(const AttnParams p
       cp_async16(dv + tile_off<D>(row, c), Vbase + off, ok ? 16 : 0);
     }
   };
-  {
+  if (!empty) {
     const uint32_t dq = smem_u32(sQ);
     for (int idx = tid; idx < TILE_M * DC; idx += kThreads) {
       const int row = idx / DC, c = idx % DC;
@@ -223,9 +225,9 @@ __global__ void __launch_bounds__(kThreads) attn_stage_kernel(const AttnParams p
       }
       cp_async16(dq + tile_off<D>(row, c), p.q + off, ok ? 16 : 0);
     }
+    load_kv(k_begin, 0);
+    cp_async_commit();
   }
-  load_kv(k_begin, 0);
-  cp_async_commit();
 
   // ---------------------------------------------------------- main loop --
   uint32_t qf[KD][4];
@@ -235,7 +237,7 @@ __global__ void __launch_bounds__(kThreads) attn_stage_kernel(const AttnParams p
   float m_a = NEG_INF, m_b = NEG_INF, l_a = 0.f, l_b = 0.f;
   const float sl2 = p.scale_log2;
 
-  const int n_blocks = ceil_div_i(k_end - k_begin, kBN);
+  const int n_blocks = empty ? 0 : ceil_div_i(k_end - k_begin, kBN);
   for (int blk = 0; blk < n_blocks; ++blk) {
     const int kb0 = k_begin + blk * kBN;
     if (blk + 1 < n_blocks) {
@@ -347,35 +349,55 @@ __global__ void __launch_bounds__(kThreads) attn_stage_kernel(const AttnParams p
   l_b += __shfl_xor_sync(0xffffffffu, l_b, 1);
   l_b += __shfl_xor_sync(0xffffffffu, l_b, 2);
 
+  // ------------------------------------------------------------ epilogue --
+  // Normalised partial of this CTA's rows: prefix stage -> its workspace
+  // slot; suffix stage -> shared memory, then merged with the other slots.
+  float *sm_m = reinterpret_cast<float *>(sK);  // [WK][TILE_M]
+  float *sm_l = sm_m + WK * TILE_M;             // [WK][TILE_M]
+  float *sm_M = sm_l + WK * TILE_M;             // [TILE_M]
+  float *sm_L = sm_M + TILE_M;                  // [TILE_M]
+  float *sm_o = sm_L + TILE_M;                  // [WK][TILE_M][D]; slice 0 = own partial
+  float *sm_lse = sm_o + WK * TILE_M * D;       // [TILE_M] own partial lse
+  float *sm_inv = sm_lse + TILE_M;              // [TILE_M]
+  float *sm_w = sm_inv + TILE_M;                // [TILE_M][kMaxSlots]
   if constexpr (WK == 1) {
     const float inv_a = l_a > 0.f ? 1.f / l_a : 0.f;
     const float inv_b = l_b > 0.f ? 1.f / l_b : 0.f;
-    if (ra < nrows) {
-      float *dst = p.o_part + out_index(ra) * D;
+    const float lse_a = l_a > 0.f ? (m_a + __log2f(l_a)) * kLn2 : NEG_INF;
+    const float lse_b = l_b > 0.f ? (m_b + __log2f(l_b)) * kLn2 : NEG_INF;
+    if constexpr (PREFIX) {
+      if (ra < nrows) {
+        float *dst = p.o_part + out_index(ra) * D;
 #pragma unroll
-      for (int dt = 0; dt < DT; ++dt)
-        *reinterpret_cast<float2 *>(dst + dt * 8 + (lane & 3) * 2) =
-            make_float2(o[dt][0] * inv_a, o[dt][1] * inv_a);
-      if ((lane & 3) == 0)
-        p.l_part[out_index(ra)] = l_a > 0.f ? (m_a + __log2f(l_a)) * kLn2 : NEG_INF;
-    }
-    if (rb < nrows) {
-      float *dst = p.o_part + out_index(rb) * D;
+        for (int dt = 0; dt < DT; ++dt)
+          *reinterpret_cast<float2 *>(dst + dt * 8 + (lane & 3) * 2) =
+              make_float2(o[dt][0] * inv_a, o[dt][1] * inv_a);
+        if ((lane & 3) == 0) p.l_part[out_index(ra)] = lse_a;
+      }
+      if (rb < nrows) {
+        float *dst = p.o_part + out_index(rb) * D;
 #pragma unroll
-      for (int dt = 0; dt < DT; ++dt)
-        *reinterpret_cast<float2 *>(dst + dt * 8 + (lane & 3) * 2) =
-            make_float2(o[dt][2] * inv_b, o[dt][3] * inv_b);
-      if ((lane & 3) == 0)
-        p.l_part[out_index(rb)] = l_b > 0.f ? (m_b + __log2f(l_b)) * kLn2 : NEG_INF;
+        for (int dt = 0; dt < DT; ++dt)
+          *reinterpret_cast<float2 *>(dst + dt * 8 + (lane & 3) * 2) =
+              make_float2(o[dt][2] * inv_b, o[dt][3] * inv_b);
+        if ((lane & 3) == 0) p.l_part[out_index(rb)] = lse_b;
+      }
+      return;
+    } else {
+#pragma unroll
+      for (int dt = 0; dt < DT; ++dt) {
+        const int d = dt * 8 + (lane & 3) * 2;
+        *reinterpret_cast<float2 *>(sm_o + ra * D + d) = make_float2(o[dt][0] * inv_a, o[dt][1] * inv_a);
+        *reinterpret_cast<float2 *>(sm_o + rb * D + d) = make_float2(o[dt][2] * inv_b, o[dt][3] * inv_b);
+      }
+      if ((lane & 3) == 0) {
+        sm_lse[ra] = lse_a;
+        sm_lse[rb] = lse_b;
+      }
     }
   } else {
-    // Combine the WK key groups of each row through shared memory (the
-    // K/V buffers are free after the loop's final barrier).
-    float *sm_m = reinterpret_cast<float *>(sK);  // [WK][TILE_M]
-    float *sm_l = sm_m + WK * TILE_M;             // [WK][TILE_M]
-    float *sm_M = sm_l + WK * TILE_M;             // [TILE_M]
-    float *sm_L = sm_M + TILE_M;                  // [TILE_M]
-    float *sm_o = sm_L + TILE_M;                  // [WK][TILE_M][D]
+    // Combine the WK key groups of each row (the K/V buffers are free after
+    // the loop's final barrier).
     if ((lane & 3) == 0) {
       sm_m[kg * TILE_M + ra] = m_a;
       sm_l[kg * TILE_M + ra] = l_a;
@@ -407,7 +429,8 @@ __global__ void __launch_bounds__(kThreads) attn_stage_kernel(const AttnParams p
       }
     }
     __syncthreads();
-    for (int idx = tid; idx < nrows * (D / 4); idx += kThreads) {
+    // sum the key groups into slice 0 (each element read and written by one thread)
+    for (int idx = tid; idx < TILE_M * (D / 4); idx += kThreads) {
       const int r = idx / (D / 4), d = (idx % (D / 4)) * 4;
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
       for (int k = 0; k < WK; ++k) {
@@ -417,11 +440,134 @@ __global__ void __launch_bounds__(kThreads) attn_stage_kernel(const AttnParams p
       const float Ls = sm_L[r];
       const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
       acc.x *= inv; acc.y *= inv; acc.z *= inv; acc.w *= inv;
-      *reinterpret_cast<float4 *>(p.o_part + out_index(r) * D + d) = acc;
+      if constexpr (PREFIX) {
+        if (r < nrows) *reinterpret_cast<float4 *>(p.o_part + out_index(r) * D + d) = acc;
+      } else {
+        *reinterpret_cast<float4 *>(sm_o + r * D + d) = acc;
+      }
     }
-    for (int r = tid; r < nrows; r += kThreads) {
+    for (int r = tid; r < TILE_M; r += kThreads) {
       const float Ls = sm_L[r];
-      p.l_part[out_index(r)] = Ls > 0.f ? (sm_M[r] + __log2f(Ls)) * kLn2 : NEG_INF;
+      const float lse_r = Ls > 0.f ? (sm_M[r] + __log2f(Ls)) * kLn2 : NEG_INF;
+      if constexpr (PREFIX) {
+        if (r < nrows) p.l_part[out_index(r)] = lse_r;
+      } else {
+        sm_lse[r] = lse_r;
+      }
+    }
+    if constexpr (PREFIX) return;
+  }
+
+  if constexpr (!PREFIX) {
+    // ---- LSE merge of this branch's rows:
+    //   out = sum_s e^{lse_s - M} O_s / sum_s e^{lse_s - M},
+    //   lse = M + ln sum_s e^{lse_s - M},  M = max_s lse_s,
+    // over the prefix splits and the suffix splits of the branch.  The union
+    // of their key ranges is exactly the branch's visible key set (Sec. 3.3),
+    // so this equals one softmax over all of it.  A partial whose range held
+    // no visible key has lse_s = -inf and weight 0.
+    __shared__ int s_last;
+    bool own_in_smem = true;
+    if (p.S_s > 1) {
+      // Several CTAs hold this branch's suffix: publish this CTA's partial;
+      // the last CTA to arrive merges them all (no CTA ever waits).
+      __syncthreads();
+      for (int idx = tid; idx < nrows * (D / 4); idx += kThreads) {
+        const int r = idx / (D / 4), d = (idx % (D / 4)) * 4;
+        *reinterpret_cast<float4 *>(p.o_part + out_index(r) * D + d) =
+            *reinterpret_cast<const float4 *>(sm_o + r * D + d);
+      }
+      for (int r = tid; r < nrows; r += kThreads) p.l_part[out_index(r)] = sm_lse[r];
+      __threadfence();
+      __syncthreads();
+      int *ctr = p.counters + (static_cast<size_t>(bidx) * p.H_kv + g) * ceil_div_i(m * G, TILE_M) +
+                 r0 / TILE_M;
+      if (tid == 0) s_last = atomicAdd(ctr, 1) == p.S_s - 1;
+      __syncthreads();
+      if (!s_last) return;
+      __threadfence();
+      if (tid == 0) atomicExch(ctr, 0);
+      own_in_smem = false;
+    }
+    __syncthreads();
+    const int n_glob = own_in_smem ? p.S_p : p.S_p + p.S_s;  // partials read from the workspace
+    auto slot_index = [&](int s, int r) -> size_t {
+      const int token = tokbase + (r0 + r) / G;
+      const int head = g * G + (r0 + r) % G;
+      return (static_cast<size_t>(s) * p.rows_total + token) * p.H_q + head;
+    };
+    // weights: one row per thread, all of the row's lse loads in flight
+    static_assert(16 * WR <= kThreads, "one thread per row");
+    if (tid < nrows) {
+      const int r = tid;
+      float ls[kMaxSlots];
+#pragma unroll
+      for (int s = 0; s < kMaxSlots; ++s)
+        ls[s] = s < n_glob ? p.l_part[slot_index(s, r)] : NEG_INF;
+      float M = own_in_smem ? sm_lse[r] : NEG_INF;
+#pragma unroll
+      for (int s = 0; s < kMaxSlots; ++s) M = fmaxf(M, ls[s]);
+      float wsum = 0.f;
+#pragma unroll
+      for (int s = 0; s < kMaxSlots; ++s) {
+        const float w = ls[s] == NEG_INF ? 0.f : __expf(ls[s] - M);
+        if (s < n_glob) sm_w[r * kMaxSlots + s] = w;
+        wsum += w;
+      }
+      const float w_own = own_in_smem && sm_lse[r] != NEG_INF ? __expf(sm_lse[r] - M) : 0.f;
+      sm_w[r * kMaxSlots + n_glob] = w_own;
+      wsum += w_own;
+      sm_inv[r] = wsum > 0.f ? 1.f / wsum : 0.f;
+      if (p.lse) p.lse[slot_index(0, r)] = M == NEG_INF ? NEG_INF : M + logf(wsum);
+    }
+    __syncthreads();
+    // outputs: each thread owns up to kElems (row, 4-column) elements and, per
+    // partial, issues all of their loads before accumulating
+    constexpr int kElems = (16 * WR * (D / 4) + kThreads - 1) / kThreads;
+    const int total = nrows * (D / 4);
+    float4 acc[kElems];
+#pragma unroll
+    for (int u = 0; u < kElems; ++u) {
+      acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      const int idx = tid + u * kThreads;
+      if (own_in_smem && idx < total) {
+        const int r = idx / (D / 4), d = (idx % (D / 4)) * 4;
+        const float w = sm_w[r * kMaxSlots + n_glob];
+        const float4 v = *reinterpret_cast<const float4 *>(sm_o + r * D + d);
+        acc[u] = make_float4(w * v.x, w * v.y, w * v.z, w * v.w);
+      }
+    }
+    for (int s = 0; s < n_glob; ++s) {
+      float4 v[kElems];
+      float w[kElems];
+#pragma unroll
+      for (int u = 0; u < kElems; ++u) {
+        const int idx = tid + u * kThreads;
+        const int r = idx / (D / 4), d = (idx % (D / 4)) * 4;
+        w[u] = idx < total ? sm_w[r * kMaxSlots + s] : 0.f;
+        v[u] = w[u] != 0.f
+                   ? *reinterpret_cast<const float4 *>(p.o_part + slot_index(s, r) * D + d)
+                   : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int u = 0; u < kElems; ++u) {
+        acc[u].x += w[u] * v[u].x;
+        acc[u].y += w[u] * v[u].y;
+        acc[u].z += w[u] * v[u].z;
+        acc[u].w += w[u] * v[u].w;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kElems; ++u) {
+      const int idx = tid + u * kThreads;
+      if (idx < total) {
+        const int r = idx / (D / 4), d = (idx % (D / 4)) * 4;
+        const float inv = sm_inv[r];
+        uint2 packed;
+        packed.x = pack_bf16x2(acc[u].x * inv, acc[u].y * inv);
+        packed.y = pack_bf16x2(acc[u].z * inv, acc[u].w * inv);
+        *reinterpret_cast<uint2 *>(p.out + slot_index(0, r) * D + d) = packed;
+      }
     }
   }
 }
@@ -430,6 +576,16 @@ template <int D, int WR, bool PREFIX>
 size_t stage_smem() {
   return static_cast<size_t>(16 * WR) * D * 2 + 2ull * 2 * kBN * D * 2;
 }
+// The epilogue scratch (per-row stats, own partial, merge weights) lives in
+// the K/V buffers.
+template <int D, int WR>
+constexpr size_t epilogue_floats() {
+  return (2 * (4 / WR) + 4) * (16 * WR) + (4 / WR) * (16 * WR) * D + (16 * WR) * kMaxSlots;
+}
+static_assert(epilogue_floats<128, 1>() * 4 <= 4 * kBN * 128 * 2, "epilogue scratch");
+static_assert(epilogue_floats<128, 4>() * 4 <= 4 * kBN * 128 * 2, "epilogue scratch");
+static_assert(epilogue_floats<64, 1>() * 4 <= 4 * kBN * 64 * 2, "epilogue scratch");
+static_assert(epilogue_floats<64, 4>() * 4 <= 4 * kBN * 64 * 2, "epilogue scratch");
 
 template <int D, int WR, bool PREFIX>
 cudaError_t launch_stage(const AttnParams &p, dim3 grid, cudaStream_t s) {

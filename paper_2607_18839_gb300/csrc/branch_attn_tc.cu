@@ -1,32 +1,45 @@
-// prefix_tc.cu -- the shared-prefix stage on 5th-generation tensor cores.
+// branch_attn_tc.cu -- the branch-attention step on 5th-generation tensor
+// cores: shared prefix and private suffixes in one kernel.
 //
-// What it computes is the shared-prefix part of each branch's attention
-// (Sec. 3.3): all query rows of a page's branches that read KV head g are
-// stacked (row r <-> token branch_cu[d]*m + r/G, query head g*G + r%G) and
-// attend to the page's prefix keys [0, P_d) -- masked per row at the
-// branch's fork-position prefix length -- producing, per key split, the
-// normalised partial output O_s (fp32) and lse_s (natural log) that the LSE
-// merge combines with the private-suffix partials.
+// What it computes (Sec. 3.3, "Dynamic Branch Forking and Efficient Context
+// Isolation"; Sec. 3.4 for the m P-MTP queries): all query rows of a page's
+// branches that read KV head g are stacked (row r <-> token
+// branch_cu[d]*m + r/G, query head g*G + r%G).  Each row attends to
+//   - the page's shared prefix keys [0, P_b), P_b its branch's fork-position
+//     prefix length (P_d when none is given), and
+//   - its own branch's private keys j <= L_b - m + i (i = the row's query).
+// The page's prefix is read once per 128 or 256 stacked rows instead of once
+// per branch: that is the shared-prefix KV reuse the method relies on.
 //
-// How: one CTA owns NT tiles of 128 stacked rows (NT = 1 or 2) and one key
-// split of one (page, KV head).  Each 128-key K / V tile is loaded once and
-// used by all NT row tiles.
-//   warp 0      TMA producer: the Q tiles once, then K and V tiles into
-//               two-stage rings (128-byte swizzled, one box per 64 columns).
-//               A K stage is refilled as soon as its Q K^T MMAs finish, a V
-//               stage once its P V MMAs finish.
+// Key blocks: a CTA walks 128-key blocks of two kinds,
+//   prefix blocks  128 consecutive prefix keys (3-D TMA box per 64 columns),
+//   suffix blocks  8 pages of 16 keys, packed from the private caches of the
+//                  CTA's branches in branch order (4-D TMA box per page).
+// For every row and block the visible columns form one interval [lo, hi):
+// a prefix block's keys below the row's limit, or the row's own branch's
+// pages up to its causal bound.  Rows of other branches see nothing of a
+// suffix page, so its probabilities are zero for them.
+//
+// How: one CTA owns NT tiles of 128 stacked rows (NT = 1 or 2) and one split
+// (an even share of the blocks) of one (page, KV head).
+//   warp 0      TMA producer: the Q tiles once, then K and V blocks into
+//               two-stage rings (128-byte swizzled).  A K stage is refilled
+//               as soon as its Q K^T MMAs finish, a V stage once its P V MMAs
+//               finish.
 //   warp 1      TMEM owner and MMA issuer (one thread):
-//                 S = Q K_j^T  -> TMEM (fp32, 128 columns per tile)
-//                 O += P_j V_j  with P_j read from TMEM (bf16, written over
-//                               S) and O accumulated in TMEM
-//               NT = 1: S is double buffered, so Q K_{j+1}^T runs while the
-//               softmax works on block j.  NT = 2: the two tiles alternate,
-//               so one tile's MMAs run while the other tile's softmax works.
+//                 S = Q K^T   -> TMEM (fp32, 128 columns per tile)
+//                 O += P V    with P read from TMEM (bf16, written over S) and
+//                             O accumulated in TMEM
+//               NT = 1: S is double buffered, so the next Q K^T runs while the
+//               softmax works.  NT = 2: the two tiles alternate, so one
+//               tile's MMAs run while the other tile's softmax works.
 //   warps 2..   softmax, one warpgroup per tile: thread t of warp w owns TMEM
 //               lane 32*(w%4)+t, i.e. one query row, so row max / sum need
 //               no shuffles.  O is rescaled in TMEM only when a row's running
 //               max grows by more than 2^8; the stale max stays exact after
 //               the final normalisation.
+// One split: the CTA writes the final bf16 output and lse.  Several splits:
+// it writes its normalised fp32 partial and lse for merge.cu.
 // All waits are bounded; a timeout sets HPD_DEVERR_TIMEOUT and the CTA
 // drains its in-flight copies and MMAs, frees its TMEM and exits.
 #include <atomic>
@@ -41,6 +54,9 @@ using tc::kBlk;
 using tc::kRows;
 
 constexpr uint32_t kTmemCols = 512;
+constexpr int kMaxCtaBranches = 258;  // branches touching 256 stacked rows, + 1
+constexpr int kPageCap = 4096;        // suffix page ids kept in shared memory
+constexpr int kPagesPerBlock = kBlk / kPage;
 
 template <int D, int NT>
 struct TcLayout {
@@ -50,7 +66,8 @@ struct TcLayout {
   static constexpr uint32_t kQ = 0;                     // NT tiles
   static constexpr uint32_t kK = NT * kTileBytes;       // 2 stages
   static constexpr uint32_t kV = kK + 2 * kTileBytes;   // 2 stages
-  static constexpr uint32_t kBytes = kV + 2 * kTileBytes;
+  static constexpr uint32_t kPages = kV + 2 * kTileBytes;  // int32 [kPageCap]
+  static constexpr uint32_t kBytes = kPages + kPageCap * 4;
   static constexpr uint32_t kDynSmem = kBytes + 1024;   // slack to align to 1024
   static constexpr int kThreads = 32 * (2 + 4 * NT);
   // TMEM columns: S of buffer / tile i at col_s(i), O of tile t at col_o(t).
@@ -70,6 +87,8 @@ struct __align__(8) TcShared {
   int abort;
   int info[4];
   int kmax;
+  int page_start[kMaxCtaBranches + 1];  // packed page offset of each CTA branch
+  int blen[kMaxCtaBranches];            // private length L_b (clamped)
 };
 
 __device__ __forceinline__ void set_abort(TcShared &sh, uint32_t *err) {
@@ -79,13 +98,16 @@ __device__ __forceinline__ void set_abort(TcShared &sh, uint32_t *err) {
 
 template <int D, int NT>
 __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
-    prefix_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
-                     const __grid_constant__ CUtensorMap tm_k,
-                     const __grid_constant__ CUtensorMap tm_v, const AttnParams p) {
+    branch_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
+                          const __grid_constant__ CUtensorMap tm_k,
+                          const __grid_constant__ CUtensorMap tm_v,
+                          const __grid_constant__ CUtensorMap tm_kc,
+                          const __grid_constant__ CUtensorMap tm_vc, const AttnParams p) {
   using L = TcLayout<D, NT>;
   extern __shared__ uint8_t smem_raw[];
   __shared__ TcShared sh;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+  int *page_tab = reinterpret_cast<int *>(smem_raw + (sbase - smem_u32(smem_raw)) + L::kPages);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int G = p.G, m = p.m;
   const int TT = kRows / G;  // tokens per 128-row tile
@@ -113,42 +135,96 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
   const int ntok = min(NT * TT, (b1 - b0) * m - lt * NT * TT);
   const int nrows = ntok * G;
   const int n_act = NT == 1 ? 1 : (nrows > kRows ? 2 : 1);  // row tiles holding rows
-  int k_begin, k_end;
-  tc::split_range(P_d, p.S_p, split, k_begin, k_end);
+  const int b_lo = tok0 / m;
+  const int nbc = (tok0 + ntok - 1) / m - b_lo + 1;  // branches of this CTA's rows
 
-  auto out_index = [&](int r) -> size_t {
-    const int token = tok0 + r / G;
-    const int head = g * G + r % G;
-    return (static_cast<size_t>(split) * p.rows_total + token) * p.H_q + head;
-  };
-  // exclusive key limit of CTA row r (fork-position prefix, split end)
-  auto row_limit = [&](int r) -> int {
-    if (r >= nrows) return k_begin;
-    int lim = k_end;
-    if (p.branch_prefix_len) {
-      const int b = (tok0 + r / G) / m;
-      int f = p.branch_prefix_len[b];
-      if (f < 0 || f > P_d) {
-        flag_error(p.err, HPD_DEVERR_FORK_LEN);
-        f = min(max(f, 0), P_d);
+  // private lengths and packed page offsets of the CTA's branches
+  if (warp == 0) {
+    int base = 0;
+    for (int c0 = 0; c0 < nbc; c0 += 32) {
+      const int bl = c0 + lane;
+      int np = 0;
+      if (bl < nbc) {
+        int Lb = p.branch_len[b_lo + bl];
+        const int cap = p.max_pages * kPage;
+        if (Lb < 0 || Lb > cap) {
+          flag_error(p.err, HPD_DEVERR_BRANCH_LEN);
+          Lb = min(max(Lb, 0), cap);
+        }
+        sh.blen[bl] = Lb;
+        np = ceil_div_i(Lb, kPage);
       }
-      lim = min(lim, f);
+      int incl = np;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += v;
+      }
+      if (bl < nbc) sh.page_start[bl] = base + incl - np;
+      base += __shfl_sync(0xffffffffu, incl, 31);
     }
-    return lim;
-  };
-  if (p.branch_prefix_len) {
-    if (tid == 0) sh.kmax = k_begin;
-    __syncthreads();
-    for (int r = tid; r < NT * kRows; r += L::kThreads) atomicMax(&sh.kmax, row_limit(r));
-    __syncthreads();
-    k_end = min(k_end, sh.kmax);
+    if (lane == 0) sh.page_start[nbc] = base;
   }
-  if (nrows <= 0) return;
-  if (k_end <= k_begin) {
-    for (int r = tid; r < nrows; r += L::kThreads) p.l_part[out_index(r)] = NEG_INF;
+  // prefix keys needed by the CTA's rows (fork-position prefixes may be short)
+  auto prefix_limit = [&](int r) -> int {
+    if (r >= nrows) return 0;
+    if (!p.branch_prefix_len) return P_d;
+    const int b = (tok0 + r / G) / m;
+    int f = p.branch_prefix_len[b];
+    if (f < 0 || f > P_d) {
+      flag_error(p.err, HPD_DEVERR_FORK_LEN);
+      f = min(max(f, 0), P_d);
+    }
+    return f;
+  };
+  if (tid == 0) sh.kmax = p.branch_prefix_len ? 0 : P_d;
+  __syncthreads();
+  if (p.branch_prefix_len)
+    for (int r = tid; r < NT * kRows; r += L::kThreads) atomicMax(&sh.kmax, prefix_limit(r));
+  const int P_s = sh.page_start[nbc];
+  // page ids of the packed suffix pages (valid ids only)
+  auto page_lookup = [&](int gp) -> int {
+    int lo = 0, hi = nbc;  // largest bl with page_start[bl] <= gp
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (sh.page_start[mid] <= gp) lo = mid; else hi = mid;
+    }
+    int pg = p.page_table[static_cast<size_t>(b_lo + lo) * p.max_pages + (gp - sh.page_start[lo])];
+    if (pg < 0 || pg >= p.num_pages) {
+      flag_error(p.err, HPD_DEVERR_PAGE_ID);
+      pg = 0;
+    }
+    return pg;
+  };
+  for (int gp = tid; gp < min(P_s, kPageCap); gp += L::kThreads) page_tab[gp] = page_lookup(gp);
+  __syncthreads();
+  const int nP = ceil_div_i(sh.kmax, kBlk);               // prefix blocks
+  const int nS = ceil_div_i(P_s, kPagesPerBlock);         // suffix blocks
+  const int N = nP + nS;
+  const int blk_lo = static_cast<int>(static_cast<long long>(split) * N / p.S_p);
+  const int blk_hi = static_cast<int>(static_cast<long long>(split + 1) * N / p.S_p);
+  const int n_blocks = blk_hi - blk_lo;
+  const bool final_out = p.S_p == 1;
+
+  // (token, head) index of CTA row r; partial slot index for several splits
+  auto pair_index = [&](int r) -> size_t {
+    return static_cast<size_t>(tok0 + r / G) * p.H_q + g * G + r % G;
+  };
+  auto slot_index = [&](int r) -> size_t {
+    return static_cast<size_t>(split) * p.rows_total * p.H_q + pair_index(r);
+  };
+  if (n_blocks <= 0) {
+    for (int r = tid; r < nrows; r += L::kThreads) {
+      if (final_out) {
+        uint4 *o = reinterpret_cast<uint4 *>(p.out + pair_index(r) * D);
+        for (int c = 0; c < D / 8; ++c) o[c] = make_uint4(0u, 0u, 0u, 0u);
+        if (p.lse) p.lse[pair_index(r)] = NEG_INF;
+      } else {
+        p.l_part[slot_index(r)] = NEG_INF;
+      }
+    }
     return;
   }
-  const int n_blocks = ceil_div_i(k_end - k_begin, kBlk);
 
   // ------------------------------------------------------------- setup --
   auto bar = [](uint64_t &b) { return smem_u32(&b); };
@@ -181,32 +257,48 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
       prefetch_tmap(&tm_q);
       prefetch_tmap(&tm_k);
       prefetch_tmap(&tm_v);
+      prefetch_tmap(&tm_kc);
+      prefetch_tmap(&tm_vc);
       mbar_arrive_expect_tx(bar(sh.q_full), NT * L::kTileBytes);
       for (int t = 0; t < NT; ++t)
         for (int c = 0; c < L::kChunks; ++c)
           tma_load_3d(sbase + L::kQ + t * L::kTileBytes + c * L::kChunkBytes, &tm_q,
                       bar(sh.q_full), c * 64, g * G, tok0 + t * TT);
+      auto page_of = [&](int gp) { return gp < kPageCap ? page_tab[gp] : page_lookup(gp); };
+      // one block of K (or V) into stage `dst`
+      auto load_block = [&](int jb, uint32_t dst, uint32_t b, const CUtensorMap *prefix_map,
+                            const CUtensorMap *page_map) {
+        mbar_arrive_expect_tx(b, L::kTileBytes);
+        if (jb < nP) {
+          for (int c = 0; c < L::kChunks; ++c)
+            tma_load_3d(dst + c * L::kChunkBytes, prefix_map, b, c * 64, g, pc0 + jb * kBlk);
+        } else {
+          const int gp0 = (jb - nP) * kPagesPerBlock;
+          for (int i = 0; i < kPagesPerBlock; ++i) {
+            // slots past the last page repeat it: finite values, never visible
+            const int pg = page_of(min(gp0 + i, P_s - 1));
+            for (int c = 0; c < L::kChunks; ++c)
+              tma_load_4d(dst + c * L::kChunkBytes + i * kPage * 128, page_map, b, c * 64, g, 0,
+                          pg);
+          }
+        }
+      };
       int issued_k = 0, issued_v = 0;
       for (int j = 0; j < n_blocks; ++j) {
         const int s = j & 1, prev = ((j >> 1) - 1) & 1;
-        const int key = pc0 + k_begin + j * kBlk;
         if (j >= 2 && (sh.abort || !mbar_wait(bar(sh.k_empty[s]), prev))) {
           set_abort(sh, p.err);
           break;
         }
-        mbar_arrive_expect_tx(bar(sh.k_full[s]), L::kTileBytes);
-        for (int c = 0; c < L::kChunks; ++c)
-          tma_load_3d(sbase + L::kK + s * L::kTileBytes + c * L::kChunkBytes, &tm_k,
-                      bar(sh.k_full[s]), c * 64, g, key);
+        load_block(blk_lo + j, sbase + L::kK + s * L::kTileBytes, bar(sh.k_full[s]), &tm_k,
+                   &tm_kc);
         issued_k = j + 1;
         if (j >= 2 && (sh.abort || !mbar_wait(bar(sh.v_empty[s]), prev))) {
           set_abort(sh, p.err);
           break;
         }
-        mbar_arrive_expect_tx(bar(sh.v_full[s]), L::kTileBytes);
-        for (int c = 0; c < L::kChunks; ++c)
-          tma_load_3d(sbase + L::kV + s * L::kTileBytes + c * L::kChunkBytes, &tm_v,
-                      bar(sh.v_full[s]), c * 64, g, key);
+        load_block(blk_lo + j, sbase + L::kV + s * L::kTileBytes, bar(sh.v_full[s]), &tm_v,
+                   &tm_vc);
         issued_v = j + 1;
       }
       // Do not leave while a copy into this CTA's shared memory is in flight.
@@ -312,7 +404,14 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
     const uint32_t t_lane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     const uint32_t o_col = L::col_o(t);
     if (t < n_act) {
-      const int lim = row_limit(row);
+      // the row's visible keys: prefix below lim_p; own branch's private
+      // keys j <= last, which start at packed page ps
+      const bool valid = row < nrows;
+      const int token = tok0 + row / G;
+      const int bl = valid ? token / m - b_lo : 0;
+      const int lim_p = prefix_limit(row);
+      const int ps = valid ? sh.page_start[bl] : 0;
+      const int last = valid ? sh.blen[bl] - m + (token - (b_lo + bl) * m) : -1;
       const float sl2 = p.scale_log2;
       float m_run = NEG_INF, l_run = 0.f;
       bool ok = true;
@@ -320,19 +419,29 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
         const int si = NT == 1 ? (j & 1) : t;  // S buffer / barrier index
         const int ph = NT == 1 ? ((j >> 1) & 1) : (j & 1);
         const uint32_t s_col = L::col_s(si);
-        if (sh.abort || !mbar_wait(bar(sh.s_full[si]), ph)) { ok = false; break; }
+        // warp-uniform outcome: the tcgen05.ld / st below are warp-collective
+        if (!__all_sync(0xffffffffu, !sh.abort && mbar_wait(bar(sh.s_full[si]), ph))) {
+          ok = false;
+          break;
+        }
         tc_fence_after();
-        uint32_t v[kBlk];
-#pragma unroll
-        for (int c = 0; c < kBlk; c += 32) tmem_ld32(t_lane + s_col + c, v + c);
-        tmem_ld_wait();
-        uint32_t pk[kBlk / 2];
-        const float alpha = tc::softmax_block(v, k_begin + j * kBlk, lim, sl2, m_run, l_run, pk);
-        tmem_st32(t_lane + s_col, pk);
-        tmem_st32(t_lane + s_col + 32, pk + 32);
+        const int jb = blk_lo + j;
+        int lo, hi;
+        if (jb < nP) {
+          lo = 0;
+          hi = lim_p - jb * kBlk;
+        } else {
+          const int off = (ps - (jb - nP) * kPagesPerBlock) * kPage;  // column of own key 0
+          lo = max(0, off);
+          hi = min(kBlk, off + last + 1);
+        }
+        const float alpha = tc::softmax_block_tmem(t_lane + s_col, lo, hi, sl2, m_run, l_run);
         // pv_done[t] completes once per block; waiting on every phase in
         // order keeps this warp at most one phase behind, so parity is exact.
-        if (j > 0 && !mbar_wait(bar(sh.pv_done[t]), (j - 1) & 1)) { ok = false; break; }
+        if (j > 0 && !__all_sync(0xffffffffu, mbar_wait(bar(sh.pv_done[t]), (j - 1) & 1))) {
+          ok = false;
+          break;
+        }
         // Rescale O (PV of block j-1 has landed) if any row of this warp needs it.
         if (__any_sync(0xffffffffu, j > 0 && alpha != 1.f)) {
           tc_fence_after();
@@ -353,25 +462,41 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
       }
       if (!ok) set_abort(sh, p.err);
       // -------------------------------------------------- epilogue --
-      if (ok && mbar_wait(bar(sh.pv_done[t]), (n_blocks - 1) & 1)) {
+      if (ok && __all_sync(0xffffffffu, mbar_wait(bar(sh.pv_done[t]), (n_blocks - 1) & 1))) {
         tc_fence_after();
         const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-        float *dst = row < nrows ? p.o_part + out_index(row) * D : nullptr;
+        const float lse = l_run > 0.f ? (m_run + __log2f(l_run)) * kLn2 : NEG_INF;
 #pragma unroll
         for (int c = 0; c < D; c += 32) {
           uint32_t o[32];
           tmem_ld32(t_lane + o_col + c, o);
           tmem_ld_wait();
-          if (dst) {
+          if (!valid) continue;
+          if (final_out) {
+            uint4 *dst = reinterpret_cast<uint4 *>(p.out + pair_index(row) * D + c);
+#pragma unroll
+            for (int e = 0; e < 32; e += 8)
+              dst[e / 8] = make_uint4(
+                  pack_bf16x2(__uint_as_float(o[e]) * inv, __uint_as_float(o[e + 1]) * inv),
+                  pack_bf16x2(__uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv),
+                  pack_bf16x2(__uint_as_float(o[e + 4]) * inv, __uint_as_float(o[e + 5]) * inv),
+                  pack_bf16x2(__uint_as_float(o[e + 6]) * inv, __uint_as_float(o[e + 7]) * inv));
+          } else {
+            float *dst = p.o_part + slot_index(row) * D + c;
 #pragma unroll
             for (int e = 0; e < 32; e += 4)
-              *reinterpret_cast<float4 *>(dst + c + e) =
+              *reinterpret_cast<float4 *>(dst + e) =
                   make_float4(__uint_as_float(o[e]) * inv, __uint_as_float(o[e + 1]) * inv,
                               __uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv);
           }
         }
-        if (dst)
-          p.l_part[out_index(row)] = l_run > 0.f ? (m_run + __log2f(l_run)) * kLn2 : NEG_INF;
+        if (valid) {
+          if (final_out) {
+            if (p.lse) p.lse[pair_index(row)] = lse;
+          } else {
+            p.l_part[slot_index(row)] = lse;
+          }
+        }
       } else if (ok) {
         set_abort(sh, p.err);
       }
@@ -389,8 +514,10 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
 template <int D, int NT>
 cudaError_t launch_tc(const AttnParams &p, const Plan &plan, cudaStream_t s) {
   using L = TcLayout<D, NT>;
-  CUtensorMap tq, tk, tv;
+  CUtensorMap tq, tk, tv, tkc, tvc;
   cudaError_t e = tc::make_prefix_maps(p, &tq, &tk, &tv);
+  if (e == cudaSuccess) e = tc::make_page_map(&tkc, p.k_cache, D, p.H_kv, p.num_pages);
+  if (e == cudaSuccess) e = tc::make_page_map(&tvc, p.v_cache, D, p.H_kv, p.num_pages);
   if (e != cudaSuccess) return e;
   static std::atomic<uint64_t> configured{0};
   int dev = 0;
@@ -398,19 +525,20 @@ cudaError_t launch_tc(const AttnParams &p, const Plan &plan, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   const uint64_t bit = 1ull << (dev & 63);
   if (!(configured.load(std::memory_order_acquire) & bit)) {
-    e = cudaFuncSetAttribute(prefix_tc_kernel<D, NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(branch_attn_tc_kernel<D, NT>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(L::kDynSmem));
     if (e != cudaSuccess) return e;
     configured.fetch_or(bit, std::memory_order_acq_rel);
   }
   const dim3 grid(plan.tiles_max, p.H_kv, plan.S_p);
-  prefix_tc_kernel<D, NT><<<grid, L::kThreads, L::kDynSmem, s>>>(tq, tk, tv, p);
+  branch_attn_tc_kernel<D, NT><<<grid, L::kThreads, L::kDynSmem, s>>>(tq, tk, tv, tkc, tvc, p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_prefix_stage_tc(const AttnParams &p, const Plan &plan, cudaStream_t s) {
+cudaError_t launch_branch_attn_tc(const AttnParams &p, const Plan &plan, cudaStream_t s) {
   if (plan.tiles_max <= 0) return cudaSuccess;
   if (plan.tc_tiles == 2)
     return p.D == 64 ? launch_tc<64, 2>(p, plan, s) : launch_tc<128, 2>(p, plan, s);

@@ -19,14 +19,15 @@ constexpr float kLn2 = 0.6931471805599453f;
 struct Plan {
   int G;           // query heads per KV head
   int rows_total;  // B * m query tokens
-  int S_p;         // key splits of the shared prefix per row tile
+  int S_p;         // key splits per row tile (tcgen05: prefix + suffix blocks)
   int S_s;         // key splits of a branch's private suffix
   int tiles_max;   // upper bound of prefix row tiles per KV head
   int wr_s;        // warps along rows in the suffix kernel (1, 2, 4)
   int rt_s;        // suffix row tiles per (branch, KV head)
-  bool use_tc;     // prefix stage on tcgen05 (G divides 128) or warp MMA
+  bool use_tc;     // whole step on tcgen05 (G divides 128) or warp MMA stages
   int tc_tiles;    // 128-row tiles per tcgen05 prefix CTA (1 or 2)
   size_t off_err;    // uint32 error word
+  size_t off_ctr;    // int32 tickets [B][H_kv][rt_s]
   size_t off_opart;  // fp32 [S_p + S_s][rows_total][H_q][D]
   size_t off_lpart;  // fp32 [S_p + S_s][rows_total][H_q]
   size_t bytes;      // total workspace bytes
@@ -51,15 +52,9 @@ struct AttnParams {
   float *o_part;
   float *l_part;
   uint32_t *err;
-};
-
-// Kernel parameters of the merge stage.
-struct MergeParams {
-  const float *o_part;
-  const float *l_part;
-  int S_total, rows_total, H_q, D;
-  __nv_bfloat16 *out;
-  float *lse;
+  int *counters;        // per (branch, KV head, row tile) arrival tickets, zero between calls
+  __nv_bfloat16 *out;   // final output, written by the suffix stage
+  float *lse;           // final lse (may be null)
 };
 
 // ------------------------------------------------------- device helpers --
@@ -123,11 +118,14 @@ __device__ __forceinline__ int ceil_div_i(int a, int b) { return (a + b - 1) / b
 // Host-side launchers (defined in the .cu files, called by hpd_api.cu).
 namespace hpd {
 cudaError_t launch_prefix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
-cudaError_t launch_prefix_stage_tc(const AttnParams &p, const Plan &plan, cudaStream_t s);
+cudaError_t launch_branch_attn_tc(const AttnParams &p, const Plan &plan, cudaStream_t s);
+cudaError_t launch_merge_splits(const AttnParams &p, cudaStream_t s);
 cudaError_t launch_suffix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
-cudaError_t launch_merge(const MergeParams &p, cudaStream_t s);
 // Remember `e` for hpd_last_cuda_error() and return HPD_ERR_CUDA.
 hpd_status record_cuda_error(cudaError_t e);
+// Leading workspace bytes that must be zero before a call (error word and
+// tickets); 0 if the scalars are invalid.
+size_t workspace_zero_bytes(const hpd_branch_attn_args *args);
 cudaError_t launch_accept(const __nv_bfloat16 *logits, const int32_t *drafts, int B, int m, int V,
                           int32_t *out_tokens, int32_t *accepted_len, cudaStream_t s);
 }  // namespace hpd

@@ -1,7 +1,7 @@
 // hpd_api.cu -- the C ABI of libhpd (include/hpd.h): host-side validation,
 // the launch plan and the workspace layout.  Every compute step runs in the
-// kernels of attn_mma.cu and merge_accept.cu; nothing here touches device
-// data.
+// kernels of branch_attn_tc.cu, merge.cu, attn_mma.cu and accept.cu; nothing
+// here touches device data.
 #include <cmath>
 #include <cstdint>
 
@@ -22,7 +22,7 @@ constexpr int kPlanSms = 152;          // SMs the split plan assumes (GB300)
 constexpr int kTargetCtas = kPlanSms * 4;  // warp-MMA prefix CTAs aimed for
 constexpr int kTcTileRows = 128;       // stacked rows of one tcgen05 prefix CTA
 constexpr int kMaxPrefixSplits = 8;
-constexpr int kSuffixSplitKeys = 1024;  // a suffix chunk holds at most ~this many keys
+constexpr int kSuffixSplitKeys = 1536;  // a suffix chunk holds at most ~this many keys
 constexpr int kMaxSuffixSplits = 8;
 
 size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
@@ -63,15 +63,26 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
     const int tile_tokens = pl.tc_tiles * (kTcTileRows / pl.G);
     const int tiles = ceil_div(static_cast<long long>(a->B) * a->m, tile_tokens);
     pl.tiles_max = tiles + a->n_docs;
-    // Key splits: the fewest waves of CTAs x blocks per CTA (+2 blocks of
-    // prologue / epilogue per CTA), for the longest page.
+    // Key splits: minimise the estimated time of the step, i.e. waves of
+    // CTAs x (blocks per CTA + 1 for prologue / epilogue) x time per block,
+    // plus, when split, the merge launch and its partial-result traffic.
+    // A CTA walks its page's prefix blocks and its branches' private pages
+    // (guessed at a quarter of the page-table width per branch).
     const long long ctas = static_cast<long long>(std::max(tiles, 1)) * a->H_kv;
-    const int nb = std::max(1, ceil_div(maxP, 128));
+    const int branches_per_cta =
+        std::max(1, (pl.tc_tiles * kTcTileRows) / std::max(1, a->m * pl.G));
+    const int nb = std::max(1, ceil_div(maxP, 128)) +
+                   ceil_div(static_cast<long long>(branches_per_cta) *
+                                std::max(1, a->max_pages_per_branch / 4), 8);
+    const double block_us = 1.3 * pl.tc_tiles;  // one 128-key block, measured order
+    const double partial_bytes =
+        static_cast<double>(a->B) * a->m * a->H_q * (a->D + 1) * sizeof(float);
     int best = 1;
-    long long best_cost = -1;
+    double best_cost = -1.0;
     for (int sp = 1; sp <= std::min(nb, kMaxPrefixSplits); ++sp) {
       const long long waves = (ctas * sp + kPlanSms - 1) / kPlanSms;
-      const long long cost = waves * (ceil_div(nb, sp) + 2);
+      double cost = static_cast<double>(waves) * (ceil_div(nb, sp) + 1) * block_us;
+      if (sp > 1) cost += 4.0 + sp * partial_bytes / 4.0e6;  // ~4 TB/s
       if (best_cost < 0 || cost < best_cost) {
         best_cost = cost;
         best = sp;
@@ -95,7 +106,8 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
   const size_t S = static_cast<size_t>(pl.S_p + pl.S_s);
   const size_t pairs = static_cast<size_t>(pl.rows_total) * a->H_q;
   pl.off_err = 0;
-  pl.off_opart = kAlign;
+  pl.off_ctr = kAlign;
+  pl.off_opart = align_up(pl.off_ctr + static_cast<size_t>(a->B) * a->H_kv * pl.rt_s * sizeof(int));
   pl.off_lpart = align_up(pl.off_opart + S * pairs * a->D * sizeof(float));
   pl.bytes = align_up(pl.off_lpart + S * pairs * sizeof(float));
   return pl;
@@ -104,6 +116,11 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
 }  // namespace
 
 hpd_status hpd::record_cuda_error(cudaError_t e) { return cuda_fail(e); }
+
+size_t hpd::workspace_zero_bytes(const hpd_branch_attn_args *a) {
+  if (check_scalars(a) != HPD_OK) return 0;
+  return make_plan(a).off_opart;
+}
 
 extern "C" {
 
@@ -115,12 +132,25 @@ size_t hpd_branch_attn_workspace_size(const hpd_branch_attn_args *args) {
 hpd_status hpd_workspace_init(void *workspace, size_t workspace_bytes, hpd_stream_t stream) {
   if (!workspace || !aligned(workspace, kAlign) || workspace_bytes < kAlign)
     return HPD_ERR_WORKSPACE;
-  const cudaError_t e = cudaMemsetAsync(workspace, 0, kAlign, reinterpret_cast<cudaStream_t>(stream));
+  const cudaError_t e =
+      cudaMemsetAsync(workspace, 0, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? HPD_OK : cuda_fail(e);
 }
 
 int hpd_branch_attn_launches(const hpd_branch_attn_args *args) {
-  return check_scalars(args) == HPD_OK ? 3 : 0;
+  if (check_scalars(args) != HPD_OK) return 0;
+  const hpd::Plan pl = make_plan(args);
+  return pl.use_tc ? (pl.S_p > 1 ? 2 : 1) : 2;
+}
+
+const char *hpd_branch_attn_kernel_name(const hpd_branch_attn_args *args, int k) {
+  if (check_scalars(args) != HPD_OK) return nullptr;
+  const hpd::Plan pl = make_plan(args);
+  static const char *tc_names[] = {"branch_attn_tc", "merge_splits"};
+  static const char *mma_names[] = {"prefix_stage", "suffix_merge"};
+  const int n = pl.use_tc ? (pl.S_p > 1 ? 2 : 1) : 2;
+  if (k < 0 || k >= n) return nullptr;
+  return pl.use_tc ? tc_names[k] : mma_names[k];
 }
 
 hpd_status hpd_branch_attn(const hpd_branch_attn_args *a, hpd_stream_t stream) {
@@ -175,6 +205,9 @@ hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t st
   p.o_part = reinterpret_cast<float *>(ws + pl.off_opart);
   p.l_part = reinterpret_cast<float *>(ws + pl.off_lpart);
   p.err = reinterpret_cast<uint32_t *>(ws + pl.off_err);
+  p.counters = reinterpret_cast<int *>(ws + pl.off_ctr);
+  p.out = static_cast<__nv_bfloat16 *>(a->out);
+  p.lse = a->lse;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   auto mark = [&](int k) -> cudaError_t {
@@ -182,24 +215,19 @@ hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t st
     return cudaEventRecordWithFlags(static_cast<cudaEvent_t>(ev[k]), s, cudaEventRecordExternal);
   };
   cudaError_t e = mark(0);
-  if (e == cudaSuccess)
-    e = pl.use_tc ? hpd::launch_prefix_stage_tc(p, pl, s) : hpd::launch_prefix_stage(p, pl, s);
-  if (e == cudaSuccess) e = mark(1);
-  if (e == cudaSuccess) e = hpd::launch_suffix_stage(p, pl, s);
-  if (e == cudaSuccess) e = mark(2);
-  if (e != cudaSuccess) return cuda_fail(e);
-
-  hpd::MergeParams mp{};
-  mp.o_part = p.o_part;
-  mp.l_part = p.l_part;
-  mp.S_total = pl.S_p + pl.S_s;
-  mp.rows_total = pl.rows_total;
-  mp.H_q = a->H_q;
-  mp.D = a->D;
-  mp.out = static_cast<__nv_bfloat16 *>(a->out);
-  mp.lse = a->lse;
-  e = hpd::launch_merge(mp, s);
-  if (e == cudaSuccess) e = mark(3);
+  if (pl.use_tc) {
+    if (e == cudaSuccess) e = hpd::launch_branch_attn_tc(p, pl, s);
+    if (e == cudaSuccess) e = mark(1);
+    if (pl.S_p > 1) {
+      if (e == cudaSuccess) e = hpd::launch_merge_splits(p, s);
+      if (e == cudaSuccess) e = mark(2);
+    }
+  } else {
+    if (e == cudaSuccess) e = hpd::launch_prefix_stage(p, pl, s);
+    if (e == cudaSuccess) e = mark(1);
+    if (e == cudaSuccess) e = hpd::launch_suffix_stage(p, pl, s);
+    if (e == cudaSuccess) e = mark(2);
+  }
   if (e != cudaSuccess) return cuda_fail(e);
   return HPD_OK;
 }

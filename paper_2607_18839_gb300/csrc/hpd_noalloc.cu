@@ -59,9 +59,10 @@ extern "C" hpd_status hpd_branch_attn_noalloc(const hpd_branch_attn_args *args,
   void *scratch = nullptr;
   cudaError_t e = scratch_address(&scratch);
   if (e != cudaSuccess) return hpd::record_cuda_error(e);
-  // The array keeps the previous call's contents; the error word and
-  // counters at its head must start at zero.
-  e = cudaMemsetAsync(scratch, 0, 256, reinterpret_cast<cudaStream_t>(stream));
+  // The array keeps the previous call's contents; the error word and the
+  // arrival tickets at its head must start at zero.
+  e = cudaMemsetAsync(scratch, 0, hpd::workspace_zero_bytes(&a),
+                      reinterpret_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return hpd::record_cuda_error(e);
   a.workspace = scratch;
   a.workspace_bytes = HPD_NOALLOC_WORKSPACE_BYTES;

@@ -1,6 +1,6 @@
 // tc_common.cuh -- pieces shared by the tcgen05 shared-prefix kernels:
-// locating a CTA's row tile, the key range of a prefix split, one 128-key
-// block of a row's online softmax, and TMA tensor-map encoding on the host.
+// locating a CTA's row tile, one 128-key block of a row's online softmax,
+// and TMA tensor-map encoding on the host.
 #pragma once
 
 #include <cudaTypedefs.h>
@@ -54,70 +54,107 @@ __device__ __forceinline__ void locate_tile(const AttnParams &p, int tile, int t
   }
 }
 
-// Key range of prefix split `split` of a page with P_d keys: the page's
-// ceil(P_d / 128) blocks are dealt out as evenly as possible.
-__device__ __forceinline__ void split_range(int P_d, int S_p, int split, int &k_begin,
-                                            int &k_end) {
-  const int nb = ceil_div_i(P_d, kBlk);
-  const int b0 = static_cast<int>(static_cast<long long>(split) * nb / S_p);
-  const int b1 = static_cast<int>(static_cast<long long>(split + 1) * nb / S_p);
-  k_begin = b0 * kBlk;
-  k_end = min(P_d, b1 * kBlk);
-}
-
 // One 128-key block of a row's online softmax (base 2, scaled scores).
-// v holds the raw scores of keys key0 .. key0+127; keys >= lim are masked.
-// Writes the bf16 probabilities relative to the (possibly stale) running
-// max into pk, updates m_run / l_run, and returns the factor by which the
-// row's accumulated output must be rescaled (1 if unchanged).
-__device__ __forceinline__ float softmax_block(uint32_t (&v)[kBlk], int key0, int lim, float sl2,
-                                               float &m_run, float &l_run,
-                                               uint32_t (&pk)[kBlk / 2]) {
+// s_addr is this thread's lane at the block's fp32 scores in TMEM; only
+// columns [lo, hi) are visible to the row.  The bf16 probabilities, relative
+// to the (possibly stale) running max, are written back over the scores as
+// 64 packed columns.  Updates m_run / l_run and returns the factor by which
+// the row's accumulated output must be rescaled (1 if unchanged).
+// Warp-collective (tcgen05.ld / st): all 32 lanes of the warp must call it
+// together.  Three paths, chosen per warp:
+//   no row of the warp sees the block   zeros, no loads
+//   every row sees all 128 columns      unrolled over the 128 scores held
+//                                       in registers
+//   otherwise                           a compact loop over 32-column chunks
+//                                       that reloads them from TMEM
+__device__ __forceinline__ float softmax_block_tmem(uint32_t s_addr, int lo, int hi, float sl2,
+                                                    float &m_run, float &l_run) {
+  using namespace sm100;
   const float NEG_INF = -__int_as_float(0x7f800000);
-  float mx8[8];
+  lo = max(lo, 0);
+  hi = min(hi, kBlk);
+  if (__all_sync(0xffffffffu, hi <= lo)) {
+    uint32_t z[16];
 #pragma unroll
-  for (int a = 0; a < 8; ++a) mx8[a] = NEG_INF;
-  const bool fast = sl2 > 0.f && key0 + kBlk <= lim;  // whole block visible
-  if (fast) {
-    // max of the raw scores, scaled afterwards (a positive scale keeps order)
+    for (int c = 0; c < 16; ++c) z[c] = 0u;
 #pragma unroll
-    for (int c = 0; c < kBlk; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(v[c]));
+    for (int ch = 0; ch < kBlk / 32; ++ch) tmem_st16(s_addr + ch * 16, z);
+    return 1.f;
+  }
+  float m_new, base, alpha, sum;
+  if (__all_sync(0xffffffffu, lo == 0 && hi == kBlk)) {
+    uint32_t v[kBlk];
+#pragma unroll
+    for (int ch = 0; ch < kBlk / 32; ++ch) tmem_ld32(s_addr + ch * 32, v + ch * 32);
+    tmem_ld_wait();
+    float mx8[8];
+#pragma unroll
+    for (int a = 0; a < 8; ++a) mx8[a] = NEG_INF;
+#pragma unroll
+    for (int c = 0; c < kBlk; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(v[c]) * sl2);
+    const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                           fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+    m_new = mx > m_run + kRescaleLog2 ? mx : m_run;
+    base = m_new == NEG_INF ? 0.f : m_new;
+    alpha = m_new == m_run ? 1.f : fast_exp2(m_run - base);
+    float sum8[8];
+#pragma unroll
+    for (int a = 0; a < 8; ++a) sum8[a] = 0.f;
+#pragma unroll
+    for (int ch = 0; ch < kBlk / 32; ++ch) {
+      uint32_t pk[16];
+#pragma unroll
+      for (int c = 0; c < 32; c += 2) {
+        const float e0 = fast_exp2(fmaf(__uint_as_float(v[ch * 32 + c]), sl2, -base));
+        const float e1 = fast_exp2(fmaf(__uint_as_float(v[ch * 32 + c + 1]), sl2, -base));
+        sum8[(c >> 1) & 7] += e0 + e1;
+        pk[c / 2] = pack_bf16x2(e0, e1);
+      }
+      tmem_st16(s_addr + ch * 16, pk);
+    }
+    sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
   } else {
+    // pass 1: max over the visible columns, chunk by chunk
+    float mx = NEG_INF;
+#pragma unroll 1
+    for (int ch = 0; ch < kBlk / 32; ++ch) {
+      uint32_t v[32];
+      tmem_ld32(s_addr + ch * 32, v);
+      tmem_ld_wait();
+      float mx4[4] = {NEG_INF, NEG_INF, NEG_INF, NEG_INF};
 #pragma unroll
-    for (int c = 0; c < kBlk; ++c) {
-      const float f = key0 + c < lim ? __uint_as_float(v[c]) * sl2 : NEG_INF;
-      v[c] = __float_as_uint(f);
-      mx8[c & 7] = fmaxf(mx8[c & 7], f);
+      for (int c = 0; c < 32; ++c) {
+        const int col = ch * 32 + c;
+        mx4[c & 3] = fmaxf(mx4[c & 3], col >= lo && col < hi ? __uint_as_float(v[c]) * sl2 : NEG_INF);
+      }
+      mx = fmaxf(mx, fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])));
+    }
+    m_new = mx > m_run + kRescaleLog2 ? mx : m_run;
+    base = m_new == NEG_INF ? 0.f : m_new;
+    alpha = m_new == m_run ? 1.f : fast_exp2(m_run - base);
+    // pass 2: probabilities; P chunk ch lands in columns [16 ch, 16 ch + 16),
+    // below the next chunk still to be read (32 ch + 32)
+    sum = 0.f;
+#pragma unroll 1
+    for (int ch = 0; ch < kBlk / 32; ++ch) {
+      uint32_t v[32], pk[16];
+      tmem_ld32(s_addr + ch * 32, v);
+      tmem_ld_wait();
+      float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int c = 0; c < 32; c += 2) {
+        const int col = ch * 32 + c;
+        const float e0 = col >= lo && col < hi
+                             ? fast_exp2(fmaf(__uint_as_float(v[c]), sl2, -base)) : 0.f;
+        const float e1 = col + 1 >= lo && col + 1 < hi
+                             ? fast_exp2(fmaf(__uint_as_float(v[c + 1]), sl2, -base)) : 0.f;
+        s4[(c >> 1) & 3] += e0 + e1;
+        pk[c / 2] = pack_bf16x2(e0, e1);
+      }
+      tmem_st16(s_addr + ch * 16, pk);
+      sum += (s4[0] + s4[1]) + (s4[2] + s4[3]);
     }
   }
-  float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-  if (fast) mx *= sl2;
-  const float m_new = mx > m_run + kRescaleLog2 ? mx : m_run;
-  const float base = m_new == NEG_INF ? 0.f : m_new;
-  const float alpha = m_new == m_run ? 1.f : fast_exp2(m_run - base);
-  float sum8[8];
-#pragma unroll
-  for (int a = 0; a < 8; ++a) sum8[a] = 0.f;
-  if (fast) {
-#pragma unroll
-    for (int c = 0; c < kBlk; c += 2) {
-      const float e0 = fast_exp2(fmaf(__uint_as_float(v[c]), sl2, -base));
-      const float e1 = fast_exp2(fmaf(__uint_as_float(v[c + 1]), sl2, -base));
-      sum8[(c >> 1) & 7] += e0 + e1;
-      pk[c / 2] = pack_bf16x2(e0, e1);
-    }
-  } else {
-#pragma unroll
-    for (int c = 0; c < kBlk; c += 2) {
-      const float e0 = fast_exp2(__uint_as_float(v[c]) - base);
-      const float e1 = fast_exp2(__uint_as_float(v[c + 1]) - base);
-      sum8[(c >> 1) & 7] += e0 + e1;
-      pk[c / 2] = pack_bf16x2(e0, e1);
-    }
-  }
-  const float sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) +
-                    ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
   l_run = l_run * alpha + sum;
   m_run = m_new;
   return alpha;
@@ -150,6 +187,25 @@ inline cudaError_t make_map(CUtensorMap *map, const void *base, uint64_t d0, uin
   const cuuint32_t es[3] = {1, 1, 1};
   const CUresult r =
       fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box,
+         es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+// 4-D bf16 tensor map over the paged cache [pages][16][H_kv][D]: one box
+// is one page of one KV head (64 columns x 1 head x 16 tokens x 1 page).
+inline cudaError_t make_page_map(CUtensorMap *map, const void *base, int D, int H_kv,
+                                 int num_pages) {
+  auto fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(H_kv),
+                              static_cast<cuuint64_t>(kPage), static_cast<cuuint64_t>(num_pages)};
+  const cuuint64_t row = static_cast<cuuint64_t>(D) * 2;
+  const cuuint64_t strides[3] = {row, row * H_kv, row * H_kv * kPage};
+  const cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(kPage), 1};
+  const cuuint32_t es[4] = {1, 1, 1, 1};
+  const CUresult r =
+      fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides, box,
          es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;

@@ -24,7 +24,7 @@ DEVERR = {0x1: "PREFIX_CU", 0x2: "BRANCH_CU", 0x4: "BRANCH_LEN", 0x8: "PAGE_ID",
 
 # Every entry point declared in include/hpd.h.
 EXPORTS = ("hpd_branch_attn_workspace_size", "hpd_workspace_init", "hpd_branch_attn",
-           "hpd_branch_attn_launches", "hpd_branch_attn_marked", "hpd_pmtp_accept", "hpd_read_errors", "hpd_status_string", "hpd_last_cuda_error",
+           "hpd_branch_attn_launches", "hpd_branch_attn_kernel_name", "hpd_branch_attn_marked", "hpd_pmtp_accept", "hpd_read_errors", "hpd_status_string", "hpd_last_cuda_error",
            "hpd_version", "hpd_branch_attn_noalloc")
 
 # Scratch bytes built into libhpd for hpd_branch_attn_noalloc.
@@ -77,6 +77,8 @@ def load(path: str = LIB_PATH):
     lib.hpd_branch_attn.argtypes = [ctypes.POINTER(hpd_branch_attn_args), P]
     lib.hpd_branch_attn_launches.restype = I
     lib.hpd_branch_attn_launches.argtypes = [ctypes.POINTER(hpd_branch_attn_args)]
+    lib.hpd_branch_attn_kernel_name.restype = ctypes.c_char_p
+    lib.hpd_branch_attn_kernel_name.argtypes = [ctypes.POINTER(hpd_branch_attn_args), I]
     lib.hpd_branch_attn_marked.restype = I
     lib.hpd_branch_attn_marked.argtypes = [ctypes.POINTER(hpd_branch_attn_args), P,
                                            ctypes.POINTER(ctypes.c_void_p)]
@@ -131,6 +133,11 @@ def hpd_branch_attn(args: hpd_branch_attn_args, stream_handle: Optional[int]) ->
 
 def hpd_branch_attn_launches(args: hpd_branch_attn_args) -> int:
     return int(load().hpd_branch_attn_launches(ctypes.byref(args)))
+
+
+def hpd_branch_attn_kernel_name(args: hpd_branch_attn_args, k: int) -> Optional[str]:
+    name = load().hpd_branch_attn_kernel_name(ctypes.byref(args), k)
+    return None if name is None else name.decode()
 
 
 def hpd_branch_attn_marked(args: hpd_branch_attn_args, stream_handle, event_handles) -> None:
