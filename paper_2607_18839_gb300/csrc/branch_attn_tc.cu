@@ -312,31 +312,33 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
     // ---------------------------------------------------- MMA issuer --
     if (lane == 0) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(kRows, kBlk, false);
-      constexpr uint32_t idesc_pv = idesc_bf16_f32(kRows, 64, true);
+      constexpr uint32_t idesc_pv = idesc_bf16_f32(kRows, D, true);
+      // Shared-memory descriptors are built once; a tile / stage / k-step
+      // offset only adds (offset >> 4) to the start-address field (bits
+      // 0-13), which cannot carry: every address stays below 256 KB.
+      const uint64_t dq0 = smem_desc_sw128(sbase + L::kQ, 16, 1024);
+      const uint64_t dk0 = smem_desc_sw128(sbase + L::kK, 16, 1024);
       // S[col] = Q_t K_j^T
       auto issue_qk = [&](int t, int j, uint32_t col) {
-        const uint32_t qb = sbase + L::kQ + t * L::kTileBytes;
-        const uint32_t kb = sbase + L::kK + (j & 1) * L::kTileBytes;
+        const uint64_t qd = dq0 + ((t * L::kTileBytes) >> 4);
+        const uint64_t kd = dk0 + (((j & 1) * L::kTileBytes) >> 4);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * L::kChunkBytes + (kk & 3) * 32;
-          mma_ss(tmem + col, smem_desc_sw128(qb + off, 16, 1024),
-                 smem_desc_sw128(kb + off, 16, 1024), idesc_qk, kk > 0);
+          const uint32_t off = ((kk >> 2) * L::kChunkBytes + (kk & 3) * 32) >> 4;
+          mma_ss(tmem + col, qd + off, kd + off, idesc_qk, kk > 0);
         }
       };
-      // O_t += P V_j with P in TMEM at column pcol.  One N = 64 MMA per
-      // 64-column V box: each reads a single 128-byte swizzle atom along N
-      // (MN-major B), 8-key groups 1024 bytes apart.
+      // O_t += P V_j with P in TMEM at column pcol: one N = D MMA per 16 keys.
+      // V is MN-major (D contiguous): 64-column swizzle atoms kChunkBytes
+      // apart along N (leading byte offset), 8-key groups 1024 bytes apart
+      // along K (stride byte offset).
+      const uint64_t dv0 = smem_desc_sw128(sbase + L::kV, L::kChunkBytes, 1024);
       auto issue_pv = [&](int t, int j, uint32_t pcol) {
-        const uint32_t vb = sbase + L::kV + (j & 1) * L::kTileBytes;
+        const uint64_t vd = dv0 + (((j & 1) * L::kTileBytes) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < kBlk / 16; ++kk) {
-#pragma unroll
-          for (int c = 0; c < L::kChunks; ++c)
-            mma_ts(tmem + L::col_o(t) + c * 64, tmem + pcol + kk * 8,
-                   smem_desc_sw128(vb + c * L::kChunkBytes + kk * 16 * 128, 16, 1024), idesc_pv,
-                   (j > 0 || kk > 0) ? 1u : 0u);
-        }
+        for (int kk = 0; kk < kBlk / 16; ++kk)
+          mma_ts(tmem + L::col_o(t), tmem + pcol + kk * 8, vd + ((kk * 16 * 128) >> 4), idesc_pv,
+                 (j > 0 || kk > 0) ? 1u : 0u);
       };
       auto wait = [&](uint64_t &b, int parity) {
         if (sh.abort || !mbar_wait(bar(b), parity)) return false;
