@@ -253,48 +253,56 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------ producer --
-    if (lane == 0) {
-      prefetch_tmap(&tm_q);
-      prefetch_tmap(&tm_k);
-      prefetch_tmap(&tm_v);
-      prefetch_tmap(&tm_kc);
-      prefetch_tmap(&tm_vc);
-      mbar_arrive_expect_tx(bar(sh.q_full), NT * L::kTileBytes);
+    // The whole warp runs this loop with warp-uniform values; one elected
+    // lane issues each copy.
+    {
+      if (lane == 0) {
+        prefetch_tmap(&tm_q);
+        prefetch_tmap(&tm_k);
+        prefetch_tmap(&tm_v);
+        prefetch_tmap(&tm_kc);
+        prefetch_tmap(&tm_vc);
+      }
+      __syncwarp();
+      mbar_arrive_expect_tx_elect(bar(sh.q_full), NT * L::kTileBytes);
       for (int t = 0; t < NT; ++t)
         for (int c = 0; c < L::kChunks; ++c)
-          tma_load_3d(sbase + L::kQ + t * L::kTileBytes + c * L::kChunkBytes, &tm_q,
-                      bar(sh.q_full), c * 64, g * G, tok0 + t * TT);
+          tma_load_3d_elect(sbase + L::kQ + t * L::kTileBytes + c * L::kChunkBytes, &tm_q,
+                            bar(sh.q_full), c * 64, g * G, tok0 + t * TT);
       auto page_of = [&](int gp) { return gp < kPageCap ? page_tab[gp] : page_lookup(gp); };
       // one block of K (or V) into stage `dst`
       auto load_block = [&](int jb, uint32_t dst, uint32_t b, const CUtensorMap *prefix_map,
                             const CUtensorMap *page_map) {
-        mbar_arrive_expect_tx(b, L::kTileBytes);
+        mbar_arrive_expect_tx_elect(b, L::kTileBytes);
         if (jb < nP) {
           for (int c = 0; c < L::kChunks; ++c)
-            tma_load_3d(dst + c * L::kChunkBytes, prefix_map, b, c * 64, g, pc0 + jb * kBlk);
+            tma_load_3d_elect(dst + c * L::kChunkBytes, prefix_map, b, c * 64, g, pc0 + jb * kBlk);
         } else {
           const int gp0 = (jb - nP) * kPagesPerBlock;
           for (int i = 0; i < kPagesPerBlock; ++i) {
             // slots past the last page repeat it: finite values, never visible
             const int pg = page_of(min(gp0 + i, P_s - 1));
             for (int c = 0; c < L::kChunks; ++c)
-              tma_load_4d(dst + c * L::kChunkBytes + i * kPage * 128, page_map, b, c * 64, g, 0,
-                          pg);
+              tma_load_4d_elect(dst + c * L::kChunkBytes + i * kPage * 128, page_map, b, c * 64, g,
+                                0, pg);
           }
         }
+      };
+      auto wait_all = [&](uint64_t &b, int parity) {
+        return __all_sync(0xffffffffu, !sh.abort && mbar_wait(bar(b), parity));
       };
       int issued_k = 0, issued_v = 0;
       for (int j = 0; j < n_blocks; ++j) {
         const int s = j & 1, prev = ((j >> 1) - 1) & 1;
-        if (j >= 2 && (sh.abort || !mbar_wait(bar(sh.k_empty[s]), prev))) {
-          set_abort(sh, p.err);
+        if (j >= 2 && !wait_all(sh.k_empty[s], prev)) {
+          if (lane == 0) set_abort(sh, p.err);
           break;
         }
         load_block(blk_lo + j, sbase + L::kK + s * L::kTileBytes, bar(sh.k_full[s]), &tm_k,
                    &tm_kc);
         issued_k = j + 1;
-        if (j >= 2 && (sh.abort || !mbar_wait(bar(sh.v_empty[s]), prev))) {
-          set_abort(sh, p.err);
+        if (j >= 2 && !wait_all(sh.v_empty[s], prev)) {
+          if (lane == 0) set_abort(sh, p.err);
           break;
         }
         load_block(blk_lo + j, sbase + L::kV + s * L::kTileBytes, bar(sh.v_full[s]), &tm_v,
@@ -310,7 +318,9 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
     }
   } else if (warp == 1) {
     // ---------------------------------------------------- MMA issuer --
-    if (lane == 0) {
+    // The whole warp runs this loop with warp-uniform values; one elected
+    // lane issues each MMA / commit (see sm100.cuh).
+    {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(kRows, kBlk, false);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(kRows, D, true);
       // Shared-memory descriptors are built once; a tile / stage / k-step
@@ -341,7 +351,7 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
                  (j > 0 || kk > 0) ? 1u : 0u);
       };
       auto wait = [&](uint64_t &b, int parity) {
-        if (sh.abort || !mbar_wait(bar(b), parity)) return false;
+        if (!__all_sync(0xffffffffu, !sh.abort && mbar_wait(bar(b), parity))) return false;
         tc_fence_after();
         return true;
       };
@@ -393,7 +403,7 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
           if (more) mma_commit(bar(sh.k_empty[s ^ 1]));
         }
       }
-      if (!ok) set_abort(sh, p.err);
+      if (!ok && lane == 0) set_abort(sh, p.err);
       // every MMA issued above has finished before TMEM is released
       mma_commit(bar(sh.mma_done));
       mbar_wait(bar(sh.mma_done), 0);
@@ -438,9 +448,14 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
           hi = min(kBlk, off + last + 1);
         }
         const float alpha = tc::softmax_block_tmem(t_lane + s_col, lo, hi, sl2, m_run, l_run);
-        // pv_done[t] completes once per block; waiting on every phase in
-        // order keeps this warp at most one phase behind, so parity is exact.
-        if (j > 0 && !__all_sync(0xffffffffu, mbar_wait(bar(sh.pv_done[t]), (j - 1) & 1))) {
+        // Before O may be rescaled, the P V MMA of block j-1 must have landed.
+        // NT = 2: this tile's S commit was issued after that MMA, and a
+        // commit fires only once every earlier MMA of the issuing thread has
+        // completed, so it has.  NT = 1: P V (j-1) is issued after Q K^T (j);
+        // wait for it, on every phase in order (at most one phase behind, so
+        // the parity test is exact).
+        if (NT == 1 && j > 0 &&
+            !__all_sync(0xffffffffu, mbar_wait(bar(sh.pv_done[t]), (j - 1) & 1))) {
           ok = false;
           break;
         }
@@ -464,6 +479,8 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
       }
       if (!ok) set_abort(sh, p.err);
       // -------------------------------------------------- epilogue --
+      // pv_done[t] has completed at least n_blocks - 1 phases (see above), so
+      // the parity wait for phase n_blocks - 1 is exact.
       if (ok && __all_sync(0xffffffffu, mbar_wait(bar(sh.pv_done[t]), (n_blocks - 1) & 1))) {
         tc_fence_after();
         const float inv = l_run > 0.f ? 1.f / l_run : 0.f;

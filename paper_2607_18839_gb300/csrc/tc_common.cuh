@@ -97,22 +97,28 @@ __device__ __forceinline__ float softmax_block_tmem(uint32_t s_addr, int lo, int
     m_new = mx > m_run + kRescaleLog2 ? mx : m_run;
     base = m_new == NEG_INF ? 0.f : m_new;
     alpha = m_new == m_run ? 1.f : fast_exp2(m_run - base);
-    float sum8[8];
+    // exponent arguments and running sums two lanes at a time (fp32x2 FMA / add)
+    const float2 sl2x2 = make_float2(sl2, sl2), nbase2 = make_float2(-base, -base);
+    float2 sum4[4];
 #pragma unroll
-    for (int a = 0; a < 8; ++a) sum8[a] = 0.f;
+    for (int a = 0; a < 4; ++a) sum4[a] = make_float2(0.f, 0.f);
 #pragma unroll
     for (int ch = 0; ch < kBlk / 32; ++ch) {
       uint32_t pk[16];
 #pragma unroll
       for (int c = 0; c < 32; c += 2) {
-        const float e0 = fast_exp2(fmaf(__uint_as_float(v[ch * 32 + c]), sl2, -base));
-        const float e1 = fast_exp2(fmaf(__uint_as_float(v[ch * 32 + c + 1]), sl2, -base));
-        sum8[(c >> 1) & 7] += e0 + e1;
-        pk[c / 2] = pack_bf16x2(e0, e1);
+        const float2 x = make_float2(__uint_as_float(v[ch * 32 + c]),
+                                     __uint_as_float(v[ch * 32 + c + 1]));
+        const float2 arg = __ffma2_rn(x, sl2x2, nbase2);
+        const float2 e = make_float2(fast_exp2(arg.x), fast_exp2(arg.y));
+        sum4[(c >> 1) & 3] = __fadd2_rn(sum4[(c >> 1) & 3], e);
+        pk[c / 2] = pack_bf16x2(e.x, e.y);
       }
       tmem_st16(s_addr + ch * 16, pk);
     }
-    sum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
+    const float2 s01 = __fadd2_rn(sum4[0], sum4[1]), s23 = __fadd2_rn(sum4[2], sum4[3]);
+    const float2 s03 = __fadd2_rn(s01, s23);
+    sum = s03.x + s03.y;
   } else {
     // pass 1: max over the visible columns, chunk by chunk
     float mx = NEG_INF;
