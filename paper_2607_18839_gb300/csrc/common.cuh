@@ -53,6 +53,8 @@ struct AttnParams {
   float *l_part;
   uint32_t *err;
   int *counters;        // per (branch, KV head, row tile) arrival tickets, zero between calls
+  int *unit_ctr;        // [2] persistent-kernel unit counter and finished-CTA count, zero between calls
+  int n_units;          // work units of the tcgen05 kernel (row tile x KV head x split)
   __nv_bfloat16 *out;   // final output, written by the suffix stage
   float *lse;           // final lse (may be null)
 };

@@ -206,6 +206,8 @@ hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t st
   p.l_part = reinterpret_cast<float *>(ws + pl.off_lpart);
   p.err = reinterpret_cast<uint32_t *>(ws + pl.off_err);
   p.counters = reinterpret_cast<int *>(ws + pl.off_ctr);
+  p.unit_ctr = reinterpret_cast<int *>(ws + pl.off_err + 8);  // header: err word, then counters
+  p.n_units = pl.tiles_max * a->H_kv * pl.S_p;
   p.out = static_cast<__nv_bfloat16 *>(a->out);
   p.lse = a->lse;
 

@@ -13,6 +13,13 @@
 namespace hpd {
 namespace tc {
 
+// max(a, b, c) in one instruction (three-input max.f32, sm_100 and later).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 constexpr int kRows = 128;  // stacked query rows of one tile (MMA M)
 constexpr int kBlk = 128;   // keys per block (MMA N of S = Q K^T)
 constexpr float kRescaleLog2 = 8.0f;  // tolerate a stale row max up to 2^8
@@ -87,13 +94,28 @@ __device__ __forceinline__ float softmax_block_tmem(uint32_t s_addr, int lo, int
 #pragma unroll
     for (int ch = 0; ch < kBlk / 32; ++ch) tmem_ld32(s_addr + ch * 32, v + ch * 32);
     tmem_ld_wait();
+    // row max with three-input max over 8 independent chains; on the raw
+    // scores when the scale is positive (it keeps the order), else scaled
     float mx8[8];
 #pragma unroll
     for (int a = 0; a < 8; ++a) mx8[a] = NEG_INF;
+    if (sl2 > 0.f) {
 #pragma unroll
-    for (int c = 0; c < kBlk; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], __uint_as_float(v[c]) * sl2);
-    const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                           fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      for (int c = 0; c < kBlk; c += 16)
+#pragma unroll
+        for (int a = 0; a < 8; ++a)
+          mx8[a] = fmax3(mx8[a], __uint_as_float(v[c + 2 * a]), __uint_as_float(v[c + 2 * a + 1]));
+    } else {
+#pragma unroll
+      for (int c = 0; c < kBlk; c += 16)
+#pragma unroll
+        for (int a = 0; a < 8; ++a)
+          mx8[a] = fmax3(mx8[a], __uint_as_float(v[c + 2 * a]) * sl2,
+                         __uint_as_float(v[c + 2 * a + 1]) * sl2);
+    }
+    float mx = fmax3(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(mx8[3], mx8[4], mx8[5]),
+                     fmaxf(mx8[6], mx8[7]));
+    if (sl2 > 0.f) mx *= sl2;
     m_new = mx > m_run + kRescaleLog2 ? mx : m_run;
     base = m_new == NEG_INF ? 0.f : m_new;
     alpha = m_new == m_run ? 1.f : fast_exp2(m_run - base);
