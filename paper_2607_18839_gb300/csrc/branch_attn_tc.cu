@@ -70,7 +70,10 @@ struct TcLayout {
   static constexpr uint32_t kPages = kV + 2 * kTileBytes;  // int32 [kPageCap]
   static constexpr uint32_t kBytes = kPages + kPageCap * 4;
   static constexpr uint32_t kDynSmem = kBytes + 1024;   // slack to align to 1024
-  static constexpr int kThreads = 32 * (2 + 4 * NT);
+  // softmax warpgroups per row tile: one tile per CTA splits every row's key
+  // columns over two warpgroups; two tiles keep one warpgroup each (registers)
+  static constexpr int kHalves = NT == 1 ? 2 : 1;
+  static constexpr int kThreads = 32 * (2 + 4 * kHalves * NT);  // producer, MMA, softmax
   // TMEM columns: S of buffer / tile i at col_s(i), O of tile t at col_o(t).
   static __device__ __forceinline__ uint32_t col_s(int i) { return i ? 128u : 0u; }
   static __device__ __forceinline__ uint32_t col_o(int t) { return t ? 384u : 256u; }
@@ -89,6 +92,10 @@ struct __align__(8) TcShared {
   int info[4];
   int kmax;
   int unit;
+  // the two column halves of every row exchange their partial row max
+  // (double buffered by block parity) and, at the end, their partial sums
+  float xmax[2][2][kRows];  // [half][block parity][row] (one-tile CTAs)
+  float xsum[2][kRows];     // [half][row]
   int page_start[kMaxCtaBranches + 1];  // packed page offset of each CTA branch
   int blen[kMaxCtaBranches];            // private length L_b (clamped)
 };
@@ -126,7 +133,7 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
       mbar_init(bar(sh.k_empty[s]), 1);
       mbar_init(bar(sh.v_empty[s]), 1);
       mbar_init(bar(sh.s_full[s]), 1);
-      mbar_init(bar(sh.p_full[s]), 4);  // one arrival per softmax warp
+      mbar_init(bar(sh.p_full[s]), 4 * L::kHalves);  // one arrival per softmax warp of the tile
       mbar_init(bar(sh.pv_done[s]), 1);
     }
     mbar_init(bar(sh.mma_done), 1);
@@ -420,12 +427,20 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
       if (!ok && lane == 0) set_abort(sh, p.err);
     } else {
       // ----------------------------------------------------- softmax --
-      const int t = (warp - 2) >> 2;  // row tile of this warpgroup
-      const int quad = warp & 3;      // TMEM lane quadrant this warp may access
-      const int row = t * kRows + quad * 32 + lane;
+      // Two warpgroups per row tile: warpgroup half h owns key columns
+      // [64 h, 64 h + 64) of every block and output columns [64 h, 64 h + 64).
+      constexpr int kH = L::kHalves;
+      const int t = (warp - 2) / (4 * kH);            // row tile
+      const int h = kH == 2 ? ((warp - 2) >> 2) & 1 : 0;  // column half
+      const int quad = warp & 3;            // TMEM lane quadrant this warp may access
+      const int r_in = quad * 32 + lane;    // row within the tile
+      const int row = t * kRows + r_in;
       const uint32_t t_lane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
-      const uint32_t o_col = L::col_o(t);
+      const uint32_t o_col = L::col_o(t) + h * (D / kH);
       const int cnt = NT == 1 ? jbase : jt[t];  // pv_done[t] phases completed before this unit
+      auto tile_sync = [&]() {
+        if (kH == 2) asm volatile("bar.sync %0, %1;" ::"r"(1 + t), "r"(256) : "memory");
+      };
       if (t < n_act) {
         // the row's visible keys: prefix below lim_p; own branch's private
         // keys j <= last, which start at packed page ps
@@ -436,7 +451,7 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
         const int ps = valid ? sh.page_start[bl] : 0;
         const int last = valid ? sh.blen[bl] - m + (token - (b_lo + bl) * m) : -1;
         const float sl2 = p.scale_log2;
-        float m_run = NEG_INF, l_run = 0.f;
+        float m_run = NEG_INF, l_half = 0.f;
         bool ok = true;
         for (int j = 0; j < n_blocks; ++j) {
           const int jg = jbase + j;
@@ -459,7 +474,15 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
             lo = max(0, off);
             hi = min(kBlk, off + last + 1);
           }
-          const float alpha = tc::softmax_block_tmem(t_lane + s_col, lo, hi, sl2, m_run, l_run);
+          const int par = j & 1;
+          auto xchg = [&](float mx) {
+            sh.xmax[h][par][r_in] = mx;
+            tile_sync();
+            return fmaxf(mx, sh.xmax[h ^ 1][par][r_in]);
+          };
+          const float alpha =
+              kH == 2 ? tc::softmax_half_tmem(t_lane + s_col, h, lo, hi, sl2, m_run, l_half, xchg)
+                      : tc::softmax_block_tmem(t_lane + s_col, lo, hi, sl2, m_run, l_half);
           // Before O may be rescaled, the P V MMA of block j-1 must have
           // landed.  NT = 2: this tile's S commit was issued after that MMA,
           // and a commit fires only once every earlier MMA of the issuing
@@ -471,11 +494,11 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
             ok = false;
             break;
           }
-          // Rescale O if any row of this warp needs it.
+          // Rescale this half's O columns if any row of this warp needs it.
           if (__any_sync(0xffffffffu, j > 0 && alpha != 1.f)) {
             tc_fence_after();
 #pragma unroll
-            for (int c = 0; c < D; c += 32) {
+            for (int c = 0; c < D / kH; c += 32) {
               uint32_t o[32];
               tmem_ld32(t_lane + o_col + c, o);
               tmem_ld_wait();
@@ -491,6 +514,14 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
         }
         if (!ok && lane == 0) set_abort(sh, p.err);
         // ------------------------------------------------ epilogue --
+        // row sum over both halves (both halves reach this point together:
+        // on a timeout, every wait of the tile's warps gives up)
+        float l_run = l_half;
+        if (kH == 2) {
+          sh.xsum[h][r_in] = l_half;
+          tile_sync();
+          l_run += sh.xsum[h ^ 1][r_in];
+        }
         // pv_done[t] has completed at least cnt + n_blocks - 1 phases (see
         // above), so the parity wait for the unit's last block is exact.
         if (ok && __all_sync(0xffffffffu,
@@ -499,13 +530,14 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
           const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
           const float lse = l_run > 0.f ? (m_run + __log2f(l_run)) * kLn2 : NEG_INF;
 #pragma unroll
-          for (int c = 0; c < D; c += 32) {
+          for (int c = 0; c < D / kH; c += 32) {
             uint32_t o[32];
             tmem_ld32(t_lane + o_col + c, o);
             tmem_ld_wait();
             if (!valid) continue;
+            const int dc = h * (D / kH) + c;  // output column
             if (final_out) {
-              uint4 *dst = reinterpret_cast<uint4 *>(p.out + pair_index(row) * D + c);
+              uint4 *dst = reinterpret_cast<uint4 *>(p.out + pair_index(row) * D + dc);
 #pragma unroll
               for (int e = 0; e < 32; e += 8)
                 dst[e / 8] = make_uint4(
@@ -514,7 +546,7 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
                     pack_bf16x2(__uint_as_float(o[e + 4]) * inv, __uint_as_float(o[e + 5]) * inv),
                     pack_bf16x2(__uint_as_float(o[e + 6]) * inv, __uint_as_float(o[e + 7]) * inv));
             } else {
-              float *dst = p.o_part + slot_index(row) * D + c;
+              float *dst = p.o_part + slot_index(row) * D + dc;
 #pragma unroll
               for (int e = 0; e < 32; e += 4)
                 *reinterpret_cast<float4 *>(dst + e) =
@@ -522,7 +554,7 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
                                 __uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv);
             }
           }
-          if (valid) {
+          if (valid && h == 0) {
             if (final_out) {
               if (p.lse) p.lse[pair_index(row)] = lse;
             } else {

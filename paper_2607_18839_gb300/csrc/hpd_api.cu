@@ -58,8 +58,12 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
     // tcgen05 stage: NT tiles of 128 stacked rows (128 / G tokens each) per
     // CTA, one CTA per SM.  Two tiles share every K / V load when pages are
     // big enough to fill them.
+    // Two tiles per CTA share each K / V load, which pays off when a page's
+    // prefix is long (measured: prefix 8,192: 1.5x faster; prefix <= 4,096:
+    // one-tile CTAs, with twice the units and a split softmax, are as fast
+    // or faster).
     const long long stacked = static_cast<long long>(a->B) * a->m * pl.G;
-    pl.tc_tiles = stacked >= 2LL * kTcTileRows * a->n_docs ? 2 : 1;
+    pl.tc_tiles = (stacked >= 2LL * kTcTileRows * a->n_docs && maxP >= 48 * 128) ? 2 : 1;
     const int tile_tokens = pl.tc_tiles * (kTcTileRows / pl.G);
     const int tiles = ceil_div(static_cast<long long>(a->B) * a->m, tile_tokens);
     pl.tiles_max = tiles + a->n_docs;

@@ -188,6 +188,115 @@ __device__ __forceinline__ float softmax_block_tmem(uint32_t s_addr, int lo, int
   return alpha;
 }
 
+// Half of one 128-key block of a row's online softmax: this thread owns the
+// 64 columns [64 h, 64 h + 64) of its row; the thread of the other half (the
+// same TMEM lane, another warpgroup) owns the rest.  s_addr is this thread's
+// lane at the block's first column; lo / hi bound the row's visible columns
+// in block coordinates.  xchg(max of my visible scaled scores) returns the
+// row max over both halves; it must synchronise the two halves, which also
+// orders every P store of either half after both have read their scores
+// (P half h lands in packed columns [32 h, 32 h + 32), over scores of half 0).
+// Both halves apply the same running max, so O's two column halves and the
+// two partial sums l_half stay consistent.  Returns the rescale factor of O.
+// Warp-collective (tcgen05.ld / st).
+template <class Xchg>
+__device__ __forceinline__ float softmax_half_tmem(uint32_t s_addr, int h, int lo, int hi,
+                                                   float sl2, float &m_run, float &l_half,
+                                                   Xchg xchg) {
+  using namespace sm100;
+  const float NEG_INF = -__int_as_float(0x7f800000);
+  constexpr int kH = kBlk / 2;
+  lo = max(lo - h * kH, 0);
+  hi = min(hi - h * kH, kH);
+  const bool all_empty = __all_sync(0xffffffffu, hi <= lo);
+  const bool all_full = __all_sync(0xffffffffu, lo == 0 && hi == kH);
+  uint32_t v[kH];
+  float mx = NEG_INF;
+  if (!all_empty) {
+    tmem_ld32(s_addr + h * kH, v);
+    tmem_ld32(s_addr + h * kH + 32, v + 32);
+    tmem_ld_wait();
+    float mx8[8];
+#pragma unroll
+    for (int a = 0; a < 8; ++a) mx8[a] = NEG_INF;
+    if (all_full && sl2 > 0.f) {
+      // raw scores: a positive scale keeps the order
+#pragma unroll
+      for (int c = 0; c < kH; c += 16)
+#pragma unroll
+        for (int a = 0; a < 8; ++a)
+          mx8[a] = fmax3(mx8[a], __uint_as_float(v[c + 2 * a]), __uint_as_float(v[c + 2 * a + 1]));
+    } else {
+#pragma unroll
+      for (int c = 0; c < kH; c += 16)
+#pragma unroll
+        for (int a = 0; a < 8; ++a) {
+          const int c0 = c + 2 * a;
+          const float x0 = c0 >= lo && c0 < hi ? __uint_as_float(v[c0]) * sl2 : NEG_INF;
+          const float x1 = c0 + 1 >= lo && c0 + 1 < hi ? __uint_as_float(v[c0 + 1]) * sl2 : NEG_INF;
+          mx8[a] = fmax3(mx8[a], x0, x1);
+        }
+    }
+    mx = fmax3(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(mx8[3], mx8[4], mx8[5]),
+               fmaxf(mx8[6], mx8[7]));
+    if (all_full && sl2 > 0.f) mx *= sl2;
+  }
+  mx = xchg(mx);
+  const float m_new = mx > m_run + kRescaleLog2 ? mx : m_run;
+  const float base = m_new == NEG_INF ? 0.f : m_new;
+  const float alpha = m_new == m_run ? 1.f : fast_exp2(m_run - base);
+  float sum = 0.f;
+  uint32_t pk[16];
+  if (all_empty) {
+#pragma unroll
+    for (int c = 0; c < 16; ++c) pk[c] = 0u;
+    tmem_st16(s_addr + h * 32, pk);
+    tmem_st16(s_addr + h * 32 + 16, pk);
+  } else {
+    const float2 sl2x2 = make_float2(sl2, sl2), nbase2 = make_float2(-base, -base);
+    float2 sum4[4];
+#pragma unroll
+    for (int a = 0; a < 4; ++a) sum4[a] = make_float2(0.f, 0.f);
+    if (all_full) {
+#pragma unroll
+      for (int ch = 0; ch < 2; ++ch) {
+#pragma unroll
+        for (int c = 0; c < 32; c += 2) {
+          const int col = ch * 32 + c;
+          const float2 x = make_float2(__uint_as_float(v[col]), __uint_as_float(v[col + 1]));
+          const float2 arg = __ffma2_rn(x, sl2x2, nbase2);
+          const float2 e = make_float2(fast_exp2(arg.x), fast_exp2(arg.y));
+          sum4[(c >> 1) & 3] = __fadd2_rn(sum4[(c >> 1) & 3], e);
+          pk[c / 2] = pack_bf16x2(e.x, e.y);
+        }
+        tmem_st16(s_addr + h * 32 + ch * 16, pk);
+      }
+    } else {
+#pragma unroll
+      for (int ch = 0; ch < 2; ++ch) {
+#pragma unroll
+        for (int c = 0; c < 32; c += 2) {
+          const int col = ch * 32 + c;
+          const float2 x = make_float2(__uint_as_float(v[col]), __uint_as_float(v[col + 1]));
+          const float2 arg = __ffma2_rn(x, sl2x2, nbase2);
+          float2 e;
+          e.x = col >= lo && col < hi ? fast_exp2(arg.x) : 0.f;
+          e.y = col + 1 >= lo && col + 1 < hi ? fast_exp2(arg.y) : 0.f;
+          sum4[(c >> 1) & 3] = __fadd2_rn(sum4[(c >> 1) & 3], e);
+          pk[c / 2] = pack_bf16x2(e.x, e.y);
+        }
+        tmem_st16(s_addr + h * 32 + ch * 16, pk);
+      }
+    }
+    const float2 s01 = __fadd2_rn(sum4[0], sum4[1]), s23 = __fadd2_rn(sum4[2], sum4[3]);
+    const float2 s03 = __fadd2_rn(s01, s23);
+    sum = s03.x + s03.y;
+  }
+  l_half = l_half * alpha + sum;
+  m_run = m_new;
+  return alpha;
+}
+
 // ------------------------------------------------------------------ host --
 inline PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
