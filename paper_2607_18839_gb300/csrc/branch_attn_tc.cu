@@ -487,15 +487,20 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
           // landed.  NT = 2: this tile's S commit was issued after that MMA,
           // and a commit fires only once every earlier MMA of the issuing
           // thread has completed, so it has.  NT = 1: P V (j-1) is issued
-          // after Q K^T (j); wait for it, on every phase in order (at most
-          // one phase behind, so the parity test is exact).
-          if (NT == 1 && j > 0 &&
+          // after Q K^T (j), so a warp that rescales waits for it.  Warps
+          // skip the wait when they do not rescale, yet the parity test stays
+          // exact: Q K^T (j) was issued after P V (j-2), so the S commit
+          // awaited above implies P V (j-2) has completed, and P V (j) needs
+          // this block's P; the barrier is in one of two consecutive phases.
+          // The last block always waits, which gives the epilogue that bound.
+          const bool rescale = __any_sync(0xffffffffu, j > 0 && alpha != 1.f);
+          if (NT == 1 && j > 0 && (rescale || j == n_blocks - 1) &&
               !__all_sync(0xffffffffu, mbar_wait(bar(sh.pv_done[t]), (cnt + j - 1) & 1))) {
             ok = false;
             break;
           }
           // Rescale this half's O columns if any row of this warp needs it.
-          if (__any_sync(0xffffffffu, j > 0 && alpha != 1.f)) {
+          if (rescale) {
             tc_fence_after();
 #pragma unroll
             for (int c = 0; c < D / kH; c += 32) {
