@@ -1,5 +1,5 @@
 // branch_attn_tc.cu -- the branch-attention step on 5th-generation tensor
-// cores: shared prefix and private suffixes in one kernel.
+// cores: shared prefix and private suffixes in one persistent kernel.
 //
 // What it computes (Sec. 3.3, "Dynamic Branch Forking and Efficient Context
 // Isolation"; Sec. 3.4 for the m P-MTP queries): all query rows of a page's
@@ -8,40 +8,48 @@
 //   - the page's shared prefix keys [0, P_b), P_b its branch's fork-position
 //     prefix length (P_d when none is given), and
 //   - its own branch's private keys j <= L_b - m + i (i = the row's query).
-// The page's prefix is read once per 128 or 256 stacked rows instead of once
-// per branch: that is the shared-prefix KV reuse the method relies on.
+// The page's prefix is read once per 128 stacked rows instead of once per
+// branch: that is the shared-prefix KV reuse the method relies on.
 //
-// Key blocks: a CTA walks 128-key blocks of two kinds,
+// Key blocks: a unit walks 128-key blocks of two kinds,
 //   prefix blocks  128 consecutive prefix keys (3-D TMA box per 64 columns),
 //   suffix blocks  8 pages of 16 keys, packed from the private caches of the
-//                  CTA's branches in branch order (4-D TMA box per page).
+//                  unit's branches in branch order (4-D TMA box per page).
 // For every row and block the visible columns form one interval [lo, hi):
 // a prefix block's keys below the row's limit, or the row's own branch's
 // pages up to its causal bound.  Rows of other branches see nothing of a
-// suffix page, so its probabilities are zero for them.
+// suffix page, so their probabilities are zero there.
 //
-// How: one CTA owns NT tiles of 128 stacked rows (NT = 1 or 2) and one split
-// (an even share of the blocks) of one (page, KV head).
-//   warp 0      TMA producer: the Q tiles once, then K and V blocks into
-//               two-stage rings (128-byte swizzled).  A K stage is refilled
-//               as soon as its Q K^T MMAs finish, a V stage once its P V MMAs
-//               finish.
-//   warp 1      TMEM owner and MMA issuer (one thread):
-//                 S = Q K^T   -> TMEM (fp32, 128 columns per tile)
-//                 O += P V    with P read from TMEM (bf16, written over S) and
-//                             O accumulated in TMEM
-//               NT = 1: S is double buffered, so the next Q K^T runs while the
-//               softmax works.  NT = 2: the two tiles alternate, so one
-//               tile's MMAs run while the other tile's softmax works.
-//   warps 2..   softmax, one warpgroup per tile: thread t of warp w owns TMEM
-//               lane 32*(w%4)+t, i.e. one query row, so row max / sum need
-//               no shuffles.  O is rescaled in TMEM only when a row's running
+// Work units: (row tile of 128 stacked rows, KV head, split), a split being
+// an even share of the tile's blocks.  One CTA per SM takes units from an
+// atomic counter, and its roles run one unit apart so that nothing drains
+// between units:
+//   warp 10     scheduler: takes the next unit and prepares its metadata
+//               (page, rows, private lengths, fork limits, packed page ids)
+//               in one of two shared-memory slots while the other is in use.
+//   warps 0, 11 TMA producers: warp 0 the unit's Q tile into one of two Q
+//               slots and its K blocks, warp 11 its V blocks, each into a
+//               two-stage ring (128-byte swizzle); a K stage is refilled as
+//               soon as its Q K^T is done, whatever the V ring waits for.
+//   warp 1      TMEM owner and MMA issuer; one global sequence of blocks
+//               across units, in the order QK(b), PV(b-1):
+//                 S = Q K^T   -> TMEM (fp32, double buffered by block)
+//                 O += P V    P read from TMEM (bf16, written over S); O in
+//                             TMEM, double buffered by unit so a unit's
+//                             epilogue overlaps the next unit's MMAs.
+//   warps 2..9  softmax: two warpgroups, each owning half of every block's
+//               128 key columns and half of O's columns; thread t of warp w
+//               owns TMEM lane 32*(w%4)+t, i.e. one query row.  The two
+//               halves of a row exchange their partial max through shared
+//               memory.  O is rescaled in TMEM only when a row's running
 //               max grows by more than 2^8; the stale max stays exact after
 //               the final normalisation.
-// One split: the CTA writes the final bf16 output and lse.  Several splits:
+// One split: the unit writes the final bf16 output and lse.  Several splits:
 // it writes its normalised fp32 partial and lse for merge.cu.
-// All waits are bounded; a timeout sets HPD_DEVERR_TIMEOUT and the CTA
-// drains its in-flight copies and MMAs, frees its TMEM and exits.
+// All waits are bounded; a timeout sets HPD_DEVERR_TIMEOUT, every role
+// leaves its loop, and the CTA drains its in-flight copies and MMAs, frees
+// its TMEM and exits.  No role waits on a hardware barrier (bar.sync) inside
+// its loop, so a role that leaves early cannot strand another.
 #include <algorithm>
 #include <atomic>
 
@@ -55,90 +63,157 @@ using tc::kBlk;
 using tc::kRows;
 
 constexpr uint32_t kTmemCols = 512;
-constexpr int kMaxCtaBranches = 258;  // branches touching 256 stacked rows, + 1
-constexpr int kPageCap = 4096;        // suffix page ids kept in shared memory
+constexpr int kMaxUnitBranches = kRows + 1;  // branches touching 128 stacked rows
+constexpr int kPageCap = 2048;               // suffix page ids kept in shared memory
 constexpr int kPagesPerBlock = kBlk / kPage;
+constexpr int kSoftmaxWarps = 8;
+constexpr int kSchedWarp = 2 + kSoftmaxWarps;
+constexpr int kVWarp = kSchedWarp + 1;
+constexpr int kThreads = 32 * (kVWarp + 1);
+// consumers of a metadata slot: two producers, MMA issuer, softmax warps
+constexpr uint32_t kMetaConsumers = 3 + kSoftmaxWarps;
+constexpr int kMaxRing = 3;  // largest Q / K / V ring
 
-template <int D, int NT>
+// Metadata of one unit, written by the scheduler warp.
+struct UnitMeta {
+  int valid;     // 0: no units left
+  int g;         // KV head
+  int split;     // split index
+  int tok0;      // first query token of the tile
+  int nrows;     // stacked rows (ntok * G)
+  int b_lo;      // first branch
+  int nbc;       // branches of the rows
+  int nP;        // prefix blocks
+  int pc0;       // first prefix token of the page
+  int blk_lo;    // first block of the split
+  int n_blocks;  // blocks of the split (> 0)
+  int pad;
+  int page_start[kMaxUnitBranches + 1];  // packed page offset of each branch
+  int blen[kMaxUnitBranches];            // private length L_b (clamped)
+  int fork[kMaxUnitBranches];            // prefix keys visible to the branch
+  int page_tab[kPageCap];                // packed suffix page ids
+};
+
+template <int D>
 struct TcLayout {
   static constexpr int kChunks = D / 64;                // 64-column (128-byte) boxes
   static constexpr uint32_t kChunkBytes = kRows * 128;  // 128 rows x 128 bytes
   static constexpr uint32_t kTileBytes = kChunks * kChunkBytes;
-  static constexpr uint32_t kQ = 0;                     // NT tiles
-  static constexpr uint32_t kK = NT * kTileBytes;       // 2 stages
-  static constexpr uint32_t kV = kK + 2 * kTileBytes;   // 2 stages
-  static constexpr uint32_t kPages = kV + 2 * kTileBytes;  // int32 [kPageCap]
-  static constexpr uint32_t kBytes = kPages + kPageCap * 4;
+  static constexpr int kQSlots = 2, kKStages = 2, kVStages = 2;
+  static constexpr uint32_t kQ = 0;
+  static constexpr uint32_t kK = kQSlots * kTileBytes;
+  static constexpr uint32_t kV = kK + kKStages * kTileBytes;
+  static constexpr uint32_t kMeta = kV + kVStages * kTileBytes;  // 2 UnitMeta slots
+  static constexpr uint32_t kBytes = kMeta + 2 * sizeof(UnitMeta);
   static constexpr uint32_t kDynSmem = kBytes + 1024;   // slack to align to 1024
-  // softmax warpgroups per row tile: one tile per CTA splits every row's key
-  // columns over two warpgroups; two tiles keep one warpgroup each (registers)
-  static constexpr int kHalves = NT == 1 ? 2 : 1;
-  static constexpr int kThreads = 32 * (2 + 4 * kHalves * NT);  // producer, MMA, softmax
-  // TMEM columns: S of buffer / tile i at col_s(i), O of tile t at col_o(t).
+  // TMEM columns: S of block buffer i at col_s(i), O of unit slot o at col_o(o)
   static __device__ __forceinline__ uint32_t col_s(int i) { return i ? 128u : 0u; }
-  static __device__ __forceinline__ uint32_t col_o(int t) { return t ? 384u : 256u; }
+  static __device__ __forceinline__ uint32_t col_o(int o) { return o ? 384u : 256u; }
 };
 
 struct __align__(8) TcShared {
-  uint64_t q_full;
-  uint64_t k_full[2], v_full[2];
-  uint64_t k_empty[2], v_empty[2];
-  uint64_t s_full[2];   // NT = 1: per S buffer; NT = 2: per tile
-  uint64_t p_full[2];   // same indexing as s_full
-  uint64_t pv_done[2];  // per tile
+  uint64_t meta_full[2], meta_empty[2];
+  uint64_t q_full[kMaxRing], q_empty[kMaxRing];
+  uint64_t k_full[kMaxRing], v_full[kMaxRing];
+  uint64_t k_empty[kMaxRing], v_empty[kMaxRing];
+  uint64_t s_full[2], p_full[2];  // per S buffer
+  uint64_t pv_done;
+  uint64_t o_full[2], o_empty[2];  // per O slot
   uint64_t mma_done;
   uint32_t tmem_base;
   int abort;
-  int info[4];
-  int kmax;
-  int unit;
-  // the two column halves of every row exchange their partial row max
-  // (double buffered by block parity) and, at the end, their partial sums
-  float xmax[2][2][kRows];  // [half][block parity][row] (one-tile CTAs)
+  // the two column halves of a row exchange their partial row max (double
+  // buffered by block parity) and, at the end of a unit, their partial sums;
+  // seq counters publish each value ([half][TMEM lane quadrant])
+  float xmax[2][2][kRows];  // [half][block parity][row]
   float xsum[2][kRows];     // [half][row]
-  int page_start[kMaxCtaBranches + 1];  // packed page offset of each CTA branch
-  int blen[kMaxCtaBranches];            // private length L_b (clamped)
+  int xseq[2][2][4];        // [max | sum][half][quadrant]
 };
 
 __device__ __forceinline__ void set_abort(TcShared &sh, uint32_t *err) {
   atomicExch(&sh.abort, 1);
   flag_error(err, HPD_DEVERR_TIMEOUT);
 }
+__device__ __forceinline__ bool aborted(const TcShared &sh) {
+  return *reinterpret_cast<const volatile int *>(&sh.abort) != 0;
+}
 
-template <int D, int NT>
-__global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
+// Publish `seq` at *flag after this warp's earlier shared-memory writes
+// (release store by lane 0 once the warp's lanes are ordered by __syncwarp).
+__device__ __forceinline__ void publish_seq(int *flag, int seq) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0)
+    asm volatile("st.release.cta.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(flag)), "r"(seq)
+                 : "memory");
+}
+__device__ __forceinline__ int load_seq(const int *flag) {
+  int v;
+  asm volatile("ld.acquire.cta.shared::cta.b32 %0, [%1];" : "=r"(v) : "r"(smem_u32(flag)) : "memory");
+  return v;
+}
+// Slow path of await_seq, out of line so that the clock read stays off the
+// fast path.
+__device__ __noinline__ bool await_seq_slow(const int *flag, int seq, const int *abort) {
+  const uint64_t t0 = globaltimer();
+  for (uint32_t i = 1; load_seq(flag) < seq; ++i)
+    if ((i & 63u) == 0 &&
+        (*reinterpret_cast<const volatile int *>(abort) || globaltimer() - t0 > kWaitLimitNs))
+      return false;
+  return true;
+}
+// Wait (bounded) until *flag >= seq, with acquire ordering; false on timeout
+// or abort.
+__device__ __forceinline__ bool await_seq(const int *flag, int seq, const TcShared &sh) {
+  return load_seq(flag) >= seq || await_seq_slow(flag, seq, &sh.abort);
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
     branch_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
                           const __grid_constant__ CUtensorMap tm_k,
                           const __grid_constant__ CUtensorMap tm_v,
                           const __grid_constant__ CUtensorMap tm_kc,
                           const __grid_constant__ CUtensorMap tm_vc, const AttnParams p) {
-  using L = TcLayout<D, NT>;
+  using L = TcLayout<D>;
   extern __shared__ uint8_t smem_raw[];
   __shared__ TcShared sh;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
-  int *page_tab = reinterpret_cast<int *>(smem_raw + (sbase - smem_u32(smem_raw)) + L::kPages);
+  UnitMeta *meta =
+      reinterpret_cast<UnitMeta *>(smem_raw + (sbase - smem_u32(smem_raw)) + L::kMeta);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int G = p.G, m = p.m;
   const int TT = kRows / G;  // tokens per 128-row tile
   const float NEG_INF = -__int_as_float(0x7f800000);
   auto bar = [](uint64_t &b) { return smem_u32(&b); };
+  // bounded wait on an mbarrier phase, warp-uniform outcome; false on abort
+  auto wait_bar = [&](uint64_t &b, int parity) {
+    return __all_sync(0xffffffffu, mbar_wait(bar(b), parity, &sh.abort));
+  };
 
   // ------------------------------------------------------ once per CTA --
   if (tid == 0) {
     sh.abort = 0;
-    mbar_init(bar(sh.q_full), 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kMaxRing; ++s) {
+      mbar_init(bar(sh.q_full[s]), 1);
+      mbar_init(bar(sh.q_empty[s]), 1);
       mbar_init(bar(sh.k_full[s]), 1);
       mbar_init(bar(sh.v_full[s]), 1);
       mbar_init(bar(sh.k_empty[s]), 1);
       mbar_init(bar(sh.v_empty[s]), 1);
-      mbar_init(bar(sh.s_full[s]), 1);
-      mbar_init(bar(sh.p_full[s]), 4 * L::kHalves);  // one arrival per softmax warp of the tile
-      mbar_init(bar(sh.pv_done[s]), 1);
     }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(bar(sh.meta_full[s]), 1);
+      mbar_init(bar(sh.meta_empty[s]), kMetaConsumers);
+      mbar_init(bar(sh.s_full[s]), 1);
+      mbar_init(bar(sh.p_full[s]), kSoftmaxWarps);
+      mbar_init(bar(sh.o_full[s]), 1);
+      mbar_init(bar(sh.o_empty[s]), kSoftmaxWarps);
+    }
+    mbar_init(bar(sh.pv_done), 1);
     mbar_init(bar(sh.mma_done), 1);
     fence_mbar_init();
   }
+  if (tid < 16) (&sh.xseq[0][0][0])[tid] = 0;
   if (warp == 1) {
     tmem_alloc(smem_u32(&sh.tmem_base), kTmemCols);
     tmem_relinquish();
@@ -148,151 +223,229 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = sh.tmem_base;
 
-  // Running counts of this CTA's work, identical in every thread; barrier
-  // phases continue from one unit to the next through them.
-  int jbase = 0;            // blocks processed (K / V stages; NT = 1: S buffers)
-  int jt[2] = {0, 0};       // blocks processed by row tile t (NT = 2)
-  int uidx = 0;             // units processed (Q loads)
-
-  // ------------------------------------------- persistent loop over units --
-  // A unit is (row tile, KV head, split); CTAs take units from an atomic
-  // counter in the workspace until none are left.
-  for (;;) {
-    __syncthreads();
-    if (tid == 0) {
-      sh.unit = atomicAdd(p.unit_ctr, 1);
-      sh.info[0] = -1;
-    }
-    __syncthreads();
-    const int u = sh.unit;
-    if (u >= p.n_units || sh.abort) break;
-    const int split = u % p.S_p;
-    const int g = (u / p.S_p) % p.H_kv;
-    const int tile = u / (p.S_p * p.H_kv);
-    if (warp == 0) tc::locate_tile(p, tile, NT * TT, sh.info);
-    __syncthreads();
-    const int d = sh.info[0];
-    if (d < 0) continue;
-    const int lt = sh.info[1], b0 = sh.info[2], b1 = sh.info[3];
-    const int a0 = p.prefix_cu[d], a1 = p.prefix_cu[d + 1];
-    if (tid == 0 && (a0 < 0 || a1 < a0 || a1 > p.prefix_tokens))
-      flag_error(p.err, HPD_DEVERR_PREFIX_CU);
-    const int pc0 = min(max(a0, 0), p.prefix_tokens);
-    const int pc1 = min(max(a1, pc0), p.prefix_tokens);
-    const int P_d = pc1 - pc0;
-    const int tok0 = b0 * m + lt * NT * TT;
-    const int ntok = min(NT * TT, (b1 - b0) * m - lt * NT * TT);
-    const int nrows = ntok * G;
-    const int n_act = NT == 1 ? 1 : (nrows > kRows ? 2 : 1);  // row tiles holding rows
-    const int b_lo = tok0 / m;
-    const int nbc = (tok0 + ntok - 1) / m - b_lo + 1;  // branches of this unit's rows
-
-    // private lengths and packed page offsets of the unit's branches
-    if (warp == 0) {
-      int base = 0;
-      for (int c0 = 0; c0 < nbc; c0 += 32) {
-        const int bl = c0 + lane;
-        int np = 0;
-        if (bl < nbc) {
-          int Lb = p.branch_len[b_lo + bl];
-          const int cap = p.max_pages * kPage;
-          if (Lb < 0 || Lb > cap) {
-            flag_error(p.err, HPD_DEVERR_BRANCH_LEN);
-            Lb = min(max(Lb, 0), cap);
+  if (warp == kSchedWarp) {
+    // ------------------------------------------------------- scheduler --
+    // Fills slot k & 1 with the k-th unit of this CTA that has keys; units
+    // without any get their output written here and are skipped.
+    for (int k = 0;; ++k) {
+      const int slot = k & 1;
+      if (k >= 2 && !wait_bar(sh.meta_empty[slot], ((k >> 1) - 1) & 1)) {
+        if (lane == 0) set_abort(sh, p.err);
+        break;
+      }
+      UnitMeta &M = meta[slot];
+      bool have = false;
+      for (;;) {
+        int u = 0;
+        if (lane == 0) u = atomicAdd(p.unit_ctr, 1);
+        u = __shfl_sync(0xffffffffu, u, 0);
+        if (u >= p.n_units || aborted(sh)) break;
+        const int split = u % p.S_p;
+        const int g = (u / p.S_p) % p.H_kv;
+        const int tile = u / (p.S_p * p.H_kv);
+        // the page owning the tile: page d has ceil(#branches(d) * m / TT) tiles
+        int d = -1, lt = 0, b0 = 0, b1 = 0;
+        for (int d0 = 0, base = 0; d0 < p.n_docs && base <= tile; d0 += 32) {
+          const int dd = d0 + lane;
+          int tiles = 0, c0 = 0, c1 = 0;
+          if (dd < p.n_docs) {
+            c0 = min(max(p.branch_cu[dd], 0), p.B);
+            c1 = min(max(p.branch_cu[dd + 1], 0), p.B);
+            if (c1 < c0) {
+              flag_error(p.err, HPD_DEVERR_BRANCH_CU);
+              c1 = c0;
+            }
+            tiles = ceil_div_i((c1 - c0) * m, TT);
           }
-          sh.blen[bl] = Lb;
-          np = ceil_div_i(Lb, kPage);
-        }
-        int incl = np;
+          int incl = tiles;
 #pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int v = __shfl_up_sync(0xffffffffu, incl, o);
-          if (lane >= o) incl += v;
+          for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+          }
+          const int excl = incl - tiles;
+          const unsigned hit =
+              __ballot_sync(0xffffffffu, tiles > 0 && tile >= base + excl && tile < base + incl);
+          if (hit) {
+            const int src = __ffs(hit) - 1;
+            d = __shfl_sync(0xffffffffu, dd, src);
+            lt = __shfl_sync(0xffffffffu, tile - base - excl, src);
+            b0 = __shfl_sync(0xffffffffu, c0, src);
+            b1 = __shfl_sync(0xffffffffu, c1, src);
+            break;
+          }
+          base += __shfl_sync(0xffffffffu, incl, 31);
         }
-        if (bl < nbc) sh.page_start[bl] = base + incl - np;
-        base += __shfl_sync(0xffffffffu, incl, 31);
-      }
-      if (lane == 0) sh.page_start[nbc] = base;
-    }
-    // prefix keys needed by the unit's rows (fork-position prefixes may be short)
-    auto prefix_limit = [&](int r) -> int {
-      if (r >= nrows) return 0;
-      if (!p.branch_prefix_len) return P_d;
-      const int b = (tok0 + r / G) / m;
-      int f = p.branch_prefix_len[b];
-      if (f < 0 || f > P_d) {
-        flag_error(p.err, HPD_DEVERR_FORK_LEN);
-        f = min(max(f, 0), P_d);
-      }
-      return f;
-    };
-    if (tid == 0) sh.kmax = p.branch_prefix_len ? 0 : P_d;
-    __syncthreads();
-    if (p.branch_prefix_len)
-      for (int r = tid; r < NT * kRows; r += L::kThreads) atomicMax(&sh.kmax, prefix_limit(r));
-    const int P_s = sh.page_start[nbc];
-    // page ids of the packed suffix pages (valid ids only)
-    auto page_lookup = [&](int gp) -> int {
-      int lo = 0, hi = nbc;  // largest bl with page_start[bl] <= gp
-      while (hi - lo > 1) {
-        const int mid = (lo + hi) >> 1;
-        if (sh.page_start[mid] <= gp) lo = mid; else hi = mid;
-      }
-      int pg = p.page_table[static_cast<size_t>(b_lo + lo) * p.max_pages + (gp - sh.page_start[lo])];
-      if (pg < 0 || pg >= p.num_pages) {
-        flag_error(p.err, HPD_DEVERR_PAGE_ID);
-        pg = 0;
-      }
-      return pg;
-    };
-    for (int gp = tid; gp < min(P_s, kPageCap); gp += L::kThreads) page_tab[gp] = page_lookup(gp);
-    __syncthreads();
-    const int nP = ceil_div_i(sh.kmax, kBlk);               // prefix blocks
-    const int nS = ceil_div_i(P_s, kPagesPerBlock);         // suffix blocks
-    const int N = nP + nS;
-    const int blk_lo = static_cast<int>(static_cast<long long>(split) * N / p.S_p);
-    const int blk_hi = static_cast<int>(static_cast<long long>(split + 1) * N / p.S_p);
-    const int n_blocks = blk_hi - blk_lo;
-    const bool final_out = p.S_p == 1;
-
-    // (token, head) index of unit row r; partial slot index for several splits
-    auto pair_index = [&](int r) -> size_t {
-      return static_cast<size_t>(tok0 + r / G) * p.H_q + g * G + r % G;
-    };
-    auto slot_index = [&](int r) -> size_t {
-      return static_cast<size_t>(split) * p.rows_total * p.H_q + pair_index(r);
-    };
-    if (n_blocks <= 0) {
-      for (int r = tid; r < nrows; r += L::kThreads) {
-        if (final_out) {
-          uint4 *o = reinterpret_cast<uint4 *>(p.out + pair_index(r) * D);
-          for (int c = 0; c < D / 8; ++c) o[c] = make_uint4(0u, 0u, 0u, 0u);
-          if (p.lse) p.lse[pair_index(r)] = NEG_INF;
-        } else {
-          p.l_part[slot_index(r)] = NEG_INF;
+        if (d < 0) continue;
+        const int a0 = p.prefix_cu[d], a1 = p.prefix_cu[d + 1];
+        if (lane == 0 && (a0 < 0 || a1 < a0 || a1 > p.prefix_tokens))
+          flag_error(p.err, HPD_DEVERR_PREFIX_CU);
+        const int pc0 = min(max(a0, 0), p.prefix_tokens);
+        const int P_d = min(max(a1, pc0), p.prefix_tokens) - pc0;
+        const int tok0 = b0 * m + lt * TT;
+        const int ntok = min(TT, (b1 - b0) * m - lt * TT);
+        const int b_lo = tok0 / m;
+        const int nbc = (tok0 + ntok - 1) / m - b_lo + 1;
+        // private lengths, packed page offsets and fork limits of the branches
+        int base = 0, kmax = 0;
+        for (int c0 = 0; c0 < nbc; c0 += 32) {
+          const int bl = c0 + lane;
+          int np = 0;
+          if (bl < nbc) {
+            int Lb = p.branch_len[b_lo + bl];
+            const int cap = p.max_pages * kPage;
+            if (Lb < 0 || Lb > cap) {
+              flag_error(p.err, HPD_DEVERR_BRANCH_LEN);
+              Lb = min(max(Lb, 0), cap);
+            }
+            int f = P_d;
+            if (p.branch_prefix_len) {
+              f = p.branch_prefix_len[b_lo + bl];
+              if (f < 0 || f > P_d) {
+                flag_error(p.err, HPD_DEVERR_FORK_LEN);
+                f = min(max(f, 0), P_d);
+              }
+            }
+            M.blen[bl] = Lb;
+            M.fork[bl] = f;
+            kmax = max(kmax, f);
+            np = ceil_div_i(Lb, kPage);
+          }
+          int incl = np;
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+          }
+          if (bl < nbc) M.page_start[bl] = base + incl - np;
+          base += __shfl_sync(0xffffffffu, incl, 31);
         }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
+        const int P_s = base;
+        if (lane == 0) M.page_start[nbc] = P_s;
+        __syncwarp();
+        // packed suffix page ids (valid ids only), four lookups in flight
+        const int n_tab = min(P_s, kPageCap);
+        for (int gp0 = 0; gp0 < n_tab; gp0 += 128) {
+          int addr[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int gp = gp0 + q * 32 + lane;
+            addr[q] = -1;
+            if (gp < n_tab) {
+              int lo = 0, hi = nbc;  // largest bl with page_start[bl] <= gp
+              while (hi - lo > 1) {
+                const int mid = (lo + hi) >> 1;
+                if (M.page_start[mid] <= gp) lo = mid; else hi = mid;
+              }
+              addr[q] = (b_lo + lo) * p.max_pages + (gp - M.page_start[lo]);
+            }
+          }
+          int pg[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) pg[q] = addr[q] >= 0 ? p.page_table[addr[q]] : 0;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            if (addr[q] < 0) continue;
+            if (pg[q] < 0 || pg[q] >= p.num_pages) {
+              flag_error(p.err, HPD_DEVERR_PAGE_ID);
+              pg[q] = 0;
+            }
+            M.page_tab[gp0 + q * 32 + lane] = pg[q];
+          }
+        }
+        const int N = ceil_div_i(kmax, kBlk) + ceil_div_i(P_s, kPagesPerBlock);
+        const int blk_lo = static_cast<int>(static_cast<long long>(split) * N / p.S_p);
+        const int blk_hi = static_cast<int>(static_cast<long long>(split + 1) * N / p.S_p);
+        const int nrows = ntok * G;
+        if (blk_hi <= blk_lo) {
+          // no key in this split: zero output (one split) or an empty partial
+          for (int r = lane; r < nrows; r += 32) {
+            const size_t pair = static_cast<size_t>(tok0 + r / G) * p.H_q + g * G + r % G;
+            if (p.S_p == 1) {
+              uint4 *o = reinterpret_cast<uint4 *>(p.out + pair * D);
+              for (int c = 0; c < D / 8; ++c) o[c] = make_uint4(0u, 0u, 0u, 0u);
+              if (p.lse) p.lse[pair] = NEG_INF;
+            } else {
+              p.l_part[static_cast<size_t>(split) * p.rows_total * p.H_q + pair] = NEG_INF;
+            }
+          }
+          continue;
+        }
+        if (lane == 0) {
+          M.g = g;
+          M.split = split;
+          M.tok0 = tok0;
+          M.nrows = nrows;
+          M.b_lo = b_lo;
+          M.nbc = nbc;
+          M.nP = ceil_div_i(kmax, kBlk);
+          M.pc0 = pc0;
+          M.blk_lo = blk_lo;
+          M.n_blocks = blk_hi - blk_lo;
+        }
+        have = true;
+        break;
       }
-      continue;
-    }
-
-    if (warp == 0) {
-      // ---------------------------------------------------- producer --
-      // The whole warp runs this loop with warp-uniform values; one elected
-      // lane issues each copy.
-      if (uidx == 0 && lane == 0) {
-        prefetch_tmap(&tm_q);
-        prefetch_tmap(&tm_k);
-        prefetch_tmap(&tm_v);
-        prefetch_tmap(&tm_kc);
-        prefetch_tmap(&tm_vc);
-      }
+      if (lane == 0) M.valid = have ? 1 : 0;
       __syncwarp();
-      mbar_arrive_expect_tx_elect(bar(sh.q_full), NT * L::kTileBytes);
-      for (int t = 0; t < NT; ++t)
+      __threadfence_block();
+      if (lane == 0) mbar_arrive(bar(sh.meta_full[slot]));
+      if (!have) break;
+    }
+  } else if (warp == 0 || warp == kVWarp) {
+    // ------------------------------------------------------- producers --
+    // The whole warp runs this loop with warp-uniform values; one elected
+    // lane issues each copy.  Warp 0: Q and K; warp kVWarp: V.
+    const bool is_k = warp == 0;
+    if (lane == 0) {
+      prefetch_tmap(&tm_q);
+      prefetch_tmap(&tm_k);
+      prefetch_tmap(&tm_v);
+      prefetch_tmap(&tm_kc);
+      prefetch_tmap(&tm_vc);
+    }
+    __syncwarp();
+    int jbase = 0, issued_k = 0, issued_v = 0, issued_q = 0;
+    bool ok = true;
+    for (int k = 0; ok; ++k) {
+      const int slot = k & 1;
+      if (!(ok = wait_bar(sh.meta_full[slot], (k >> 1) & 1))) break;
+      const UnitMeta &M = meta[slot];
+      if (!M.valid) break;
+      const int g = M.g, nP = M.nP, pc0 = M.pc0, blk_lo = M.blk_lo, nb = M.n_blocks;
+      const int P_s = M.page_start[M.nbc];
+      // Q tile into slot k % kQSlots, once the Q K^T MMAs of the unit that
+      // used it last are done
+      if (is_k) {
+        const int qs = k % L::kQSlots;
+        if (k >= L::kQSlots &&
+            !(ok = wait_bar(sh.q_empty[qs], ((k / L::kQSlots) - 1) & 1)))
+          break;
+        mbar_arrive_expect_tx_elect(bar(sh.q_full[qs]), L::kTileBytes);
         for (int c = 0; c < L::kChunks; ++c)
-          tma_load_3d_elect(sbase + L::kQ + t * L::kTileBytes + c * L::kChunkBytes, &tm_q,
-                            bar(sh.q_full), c * 64, g * G, tok0 + t * TT);
-      auto page_of = [&](int gp) { return gp < kPageCap ? page_tab[gp] : page_lookup(gp); };
+          tma_load_3d_elect(sbase + L::kQ + qs * L::kTileBytes + c * L::kChunkBytes, &tm_q,
+                            bar(sh.q_full[qs]), c * 64, g * G, M.tok0);
+        issued_q = k + 1;
+      }
+      // page id of packed suffix page gp (past the shared-memory table: looked
+      // up again; an id out of range was flagged by the scheduler)
+      auto page_of = [&](int gp) -> int {
+        if (gp < kPageCap) return M.page_tab[gp];
+        int lo = 0, hi = M.nbc;
+        while (hi - lo > 1) {
+          const int mid = (lo + hi) >> 1;
+          if (M.page_start[mid] <= gp) lo = mid; else hi = mid;
+        }
+        const int pg = p.page_table[static_cast<size_t>(M.b_lo + lo) * p.max_pages +
+                                    (gp - M.page_start[lo])];
+        if (pg < 0 || pg >= p.num_pages) {
+          flag_error(p.err, HPD_DEVERR_PAGE_ID);
+          return 0;
+        }
+        return pg;
+      };
       // one block of K (or V) into stage `dst`
       auto load_block = [&](int jb, uint32_t dst, uint32_t b, const CUtensorMap *prefix_map,
                             const CUtensorMap *page_map) {
@@ -311,274 +464,262 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
           }
         }
       };
-      auto wait_all = [&](uint64_t &b, int parity) {
-        return __all_sync(0xffffffffu, !sh.abort && mbar_wait(bar(b), parity));
-      };
-      int issued_k = 0, issued_v = 0;
-      for (int j = 0; j < n_blocks; ++j) {
-        const int jg = jbase + j, s = jg & 1, prev = ((jg >> 1) - 1) & 1;
-        if (jg >= 2 && !wait_all(sh.k_empty[s], prev)) {
-          if (lane == 0) set_abort(sh, p.err);
-          break;
+      for (int j = 0; j < nb; ++j) {
+        const int jg = jbase + j;
+        if (is_k) {
+          const int s = jg % L::kKStages;
+          if (jg >= L::kKStages &&
+              !(ok = wait_bar(sh.k_empty[s], ((jg / L::kKStages) - 1) & 1)))
+            break;
+          load_block(blk_lo + j, sbase + L::kK + s * L::kTileBytes, bar(sh.k_full[s]), &tm_k,
+                     &tm_kc);
+          issued_k = jg + 1;
+        } else {
+          const int s = jg % L::kVStages;
+          if (jg >= L::kVStages &&
+              !(ok = wait_bar(sh.v_empty[s], ((jg / L::kVStages) - 1) & 1)))
+            break;
+          load_block(blk_lo + j, sbase + L::kV + s * L::kTileBytes, bar(sh.v_full[s]), &tm_v,
+                     &tm_vc);
+          issued_v = jg + 1;
         }
-        load_block(blk_lo + j, sbase + L::kK + s * L::kTileBytes, bar(sh.k_full[s]), &tm_k,
-                   &tm_kc);
-        issued_k = j + 1;
-        if (jg >= 2 && !wait_all(sh.v_empty[s], prev)) {
-          if (lane == 0) set_abort(sh, p.err);
-          break;
-        }
-        load_block(blk_lo + j, sbase + L::kV + s * L::kTileBytes, bar(sh.v_full[s]), &tm_v,
-                   &tm_vc);
-        issued_v = j + 1;
       }
-      // Do not go on while a copy into this CTA's shared memory is in flight.
-      mbar_wait(bar(sh.q_full), uidx & 1);
-      for (int j = max(0, issued_k - 2); j < issued_k; ++j)
-        mbar_wait(bar(sh.k_full[(jbase + j) & 1]), ((jbase + j) >> 1) & 1);
-      for (int j = max(0, issued_v - 2); j < issued_v; ++j)
-        mbar_wait(bar(sh.v_full[(jbase + j) & 1]), ((jbase + j) >> 1) & 1);
-    } else if (warp == 1) {
-      // ---------------------------------------------------- MMA issuer --
-      // The whole warp runs this loop with warp-uniform values; one elected
-      // lane issues each MMA / commit (see sm100.cuh).
-      constexpr uint32_t idesc_qk = idesc_bf16_f32(kRows, kBlk, false);
-      constexpr uint32_t idesc_pv = idesc_bf16_f32(kRows, D, true);
-      // Shared-memory descriptors: a tile / stage / k-step offset only adds
-      // (offset >> 4) to the start-address field (bits 0-13), which cannot
-      // carry: every address stays below 256 KB.
-      const uint64_t dq0 = smem_desc_sw128(sbase + L::kQ, 16, 1024);
-      const uint64_t dk0 = smem_desc_sw128(sbase + L::kK, 16, 1024);
-      // S[col] = Q_t K^T of global block jg
-      auto issue_qk = [&](int t, int jg, uint32_t col) {
-        const uint64_t qd = dq0 + ((t * L::kTileBytes) >> 4);
-        const uint64_t kd = dk0 + (((jg & 1) * L::kTileBytes) >> 4);
+      if (!ok) break;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(sh.meta_empty[slot]));
+      jbase += nb;
+    }
+    if (!ok && lane == 0) set_abort(sh, p.err);
+    // Do not exit while a copy into this CTA's shared memory is in flight:
+    // wait for the most recent phase of every barrier a copy may complete.
+    for (int q = max(0, issued_q - L::kQSlots); q < issued_q; ++q)
+      mbar_wait(bar(sh.q_full[q % L::kQSlots]), (q / L::kQSlots) & 1);
+    for (int jg = max(0, issued_k - L::kKStages); jg < issued_k; ++jg)
+      mbar_wait(bar(sh.k_full[jg % L::kKStages]), (jg / L::kKStages) & 1);
+    for (int jg = max(0, issued_v - L::kVStages); jg < issued_v; ++jg)
+      mbar_wait(bar(sh.v_full[jg % L::kVStages]), (jg / L::kVStages) & 1);
+  } else if (warp == 1) {
+    // ------------------------------------------------------ MMA issuer --
+    // The whole warp runs this loop with warp-uniform values; one elected
+    // lane issues each MMA / commit (see sm100.cuh).
+    constexpr uint32_t idesc_qk = idesc_bf16_f32(kRows, kBlk, false);
+    constexpr uint32_t idesc_pv = idesc_bf16_f32(kRows, D, true);
+    // Shared-memory descriptors: a slot / stage / k-step offset only adds
+    // (offset >> 4) to the start-address field (bits 0-13), which cannot
+    // carry: every address stays below 256 KB.
+    const uint64_t dq0 = smem_desc_sw128(sbase + L::kQ, 16, 1024);
+    const uint64_t dk0 = smem_desc_sw128(sbase + L::kK, 16, 1024);
+    // S[col] = Q (slot qs) K^T of global block jg
+    auto issue_qk = [&](int qs, int jg, uint32_t col) {
+      const uint64_t qd = dq0 + ((qs * L::kTileBytes) >> 4);
+      const uint64_t kd = dk0 + (((jg % L::kKStages) * L::kTileBytes) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = ((kk >> 2) * L::kChunkBytes + (kk & 3) * 32) >> 4;
-          mma_ss(tmem + col, qd + off, kd + off, idesc_qk, kk > 0);
-        }
-      };
-      // O_t (+)= P V of global block jg, P in TMEM at column pcol: one N = D
-      // MMA per 16 keys.  V is MN-major (D contiguous): 64-column swizzle
-      // atoms kChunkBytes apart along N (leading byte offset), 8-key groups
-      // 1024 bytes apart along K (stride byte offset).
-      const uint64_t dv0 = smem_desc_sw128(sbase + L::kV, L::kChunkBytes, 1024);
-      auto issue_pv = [&](int t, int jg, bool first, uint32_t pcol) {
-        const uint64_t vd = dv0 + (((jg & 1) * L::kTileBytes) >> 4);
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t off = ((kk >> 2) * L::kChunkBytes + (kk & 3) * 32) >> 4;
+        mma_ss(tmem + col, qd + off, kd + off, idesc_qk, kk > 0);
+      }
+    };
+    // O (slot os) (+)= P V of global block jg, P in TMEM at column pcol: one
+    // N = D MMA per 16 keys.  V is MN-major (D contiguous): 64-column swizzle
+    // atoms kChunkBytes apart along N (leading byte offset), 8-key groups
+    // 1024 bytes apart along K (stride byte offset).
+    const uint64_t dv0 = smem_desc_sw128(sbase + L::kV, L::kChunkBytes, 1024);
+    auto issue_pv = [&](int os, int jg, bool first, uint32_t pcol) {
+      const uint64_t vd = dv0 + (((jg % L::kVStages) * L::kTileBytes) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < kBlk / 16; ++kk)
-          mma_ts(tmem + L::col_o(t), tmem + pcol + kk * 8, vd + ((kk * 16 * 128) >> 4), idesc_pv,
-                 (!first || kk > 0) ? 1u : 0u);
-      };
-      auto wait = [&](uint64_t &b, int parity) {
-        if (!__all_sync(0xffffffffu, !sh.abort && mbar_wait(bar(b), parity))) return false;
+      for (int kk = 0; kk < kBlk / 16; ++kk)
+        mma_ts(tmem + L::col_o(os), tmem + pcol + kk * 8, vd + ((kk * 16 * 128) >> 4), idesc_pv,
+               (!first || kk > 0) ? 1u : 0u);
+    };
+    auto wait = [&](uint64_t &b, int parity) {
+      if (!wait_bar(b, parity)) return false;
+      tc_fence_after();
+      return true;
+    };
+    // The P V of a block is issued after the Q K^T of the next block (QK(b),
+    // PV(b-1)), across unit boundaries too.
+    struct Pending {
+      int jg, unit;
+      bool first, last;
+    };
+    Pending pend{0, 0, false, false};
+    bool has_pend = false;
+    auto do_pv = [&](const Pending &x) -> bool {
+      const int s = x.jg & 1, os = x.unit & 1, sv = x.jg % L::kVStages;
+      if (!wait(sh.p_full[s], (x.jg >> 1) & 1) || !wait(sh.v_full[sv], (x.jg / L::kVStages) & 1))
+        return false;
+      // O slot os last held unit x.unit - 2, whose epilogue must have read it
+      if (x.first && x.unit >= 2 && !wait(sh.o_empty[os], ((x.unit >> 1) - 1) & 1)) return false;
+      issue_pv(os, x.jg, x.first, L::col_s(s));
+      mma_commit(bar(sh.pv_done));
+      mma_commit(bar(sh.v_empty[sv]));
+      if (x.last) mma_commit(bar(sh.o_full[os]));
+      return true;
+    };
+    int jbase = 0;
+    bool ok = true;
+    for (int k = 0; ok; ++k) {
+      const int slot = k & 1;
+      if (!(ok = wait(sh.meta_full[slot], (k >> 1) & 1))) break;
+      const bool valid = meta[slot].valid != 0;
+      const int nb = meta[slot].n_blocks;
+      __syncwarp();
+      if (!valid) break;
+      if (lane == 0) mbar_arrive(bar(sh.meta_empty[slot]));
+      const int qs = k % L::kQSlots;
+      if (!(ok = wait(sh.q_full[qs], (k / L::kQSlots) & 1))) break;
+      for (int j = 0; j < nb; ++j) {
+        const int jg = jbase + j, s = jg & 1, sk = jg % L::kKStages;
+        if (!(ok = wait(sh.k_full[sk], (jg / L::kKStages) & 1))) break;
+        issue_qk(qs, jg, L::col_s(s));
+        mma_commit(bar(sh.s_full[s]));
+        mma_commit(bar(sh.k_empty[sk]));
+        if (j == nb - 1) mma_commit(bar(sh.q_empty[qs]));
+        if (has_pend && !(ok = do_pv(pend))) break;
+        pend = Pending{jg, k, j == 0, j == nb - 1};
+        has_pend = true;
+      }
+      jbase += nb;
+    }
+    if (ok && has_pend) ok = do_pv(pend);
+    if (!ok && lane == 0) set_abort(sh, p.err);
+  } else {
+    // --------------------------------------------------------- softmax --
+    // Warpgroup half h owns key columns [64 h, 64 h + 64) of every block and
+    // output columns [64 h, 64 h + 64).
+    const int h = (warp - 2) >> 2;        // column half
+    const int quad = warp & 3;            // TMEM lane quadrant this warp may access
+    const int r_in = quad * 32 + lane;    // row within the tile
+    const uint32_t t_lane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    const float sl2 = p.scale_log2;
+    int jbase = 0;
+    bool ok = true;
+    for (int k = 0; ok; ++k) {
+      const int slot = k & 1;
+      if (!(ok = wait_bar(sh.meta_full[slot], (k >> 1) & 1))) break;
+      const UnitMeta &M = meta[slot];
+      if (!M.valid) break;
+      const int g = M.g, split = M.split, tok0 = M.tok0, nb = M.n_blocks;
+      const int blk_lo = M.blk_lo, nP = M.nP;
+      // the row's visible keys: prefix below lim_p; own branch's private
+      // keys j <= last, which start at packed page ps
+      const bool valid = r_in < M.nrows;
+      const int token = tok0 + r_in / G;
+      const int bl = valid ? token / m - M.b_lo : 0;
+      const int lim_p = valid ? M.fork[bl] : 0;
+      const int ps = valid ? M.page_start[bl] : 0;
+      const int last = valid ? M.blen[bl] - m + (token - (M.b_lo + bl) * m) : -1;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(sh.meta_empty[slot]));
+      const uint32_t o_col = L::col_o(slot) + h * (D / 2);
+      float m_run = NEG_INF, l_half = 0.f;
+      for (int j = 0; j < nb; ++j) {
+        const int jg = jbase + j;
+        const int si = jg & 1;
+        // warp-uniform outcome: the tcgen05.ld / st below are warp-collective
+        if (!(ok = wait_bar(sh.s_full[si], (jg >> 1) & 1))) break;
         tc_fence_after();
-        return true;
-      };
-      bool ok = wait(sh.q_full, uidx & 1);
-      if constexpr (NT == 1) {
-        for (int j = 0; ok && j <= n_blocks; ++j) {
-          if (j < n_blocks) {
-            const int jg = jbase + j, s = jg & 1;
-            if (!(ok = wait(sh.k_full[s], (jg >> 1) & 1))) break;
-            issue_qk(0, jg, L::col_s(s));
-            mma_commit(bar(sh.s_full[s]));
-            mma_commit(bar(sh.k_empty[s]));
-          }
-          if (j >= 1) {
-            const int jg = jbase + j - 1, s = jg & 1;
-            if (!(ok = wait(sh.p_full[s], (jg >> 1) & 1) && wait(sh.v_full[s], (jg >> 1) & 1)))
-              break;
-            issue_pv(0, jg, j == 1, L::col_s(s));
-            mma_commit(bar(sh.pv_done[0]));
-            mma_commit(bar(sh.v_empty[s]));
-          }
+        const int jb = blk_lo + j;
+        int lo, hi;
+        if (jb < nP) {
+          lo = 0;
+          hi = lim_p - jb * kBlk;
+        } else {
+          const int off = (ps - (jb - nP) * kPagesPerBlock) * kPage;  // column of own key 0
+          lo = max(0, off);
+          hi = min(kBlk, off + last + 1);
         }
-      } else {
-        // tile t's S lives at col_s(t); tiles alternate on the tensor pipe:
-        //   PV_0(j)  QK_0(j+1)  PV_1(j)  QK_1(j+1)  ...
-        if (ok && (ok = wait(sh.k_full[jbase & 1], (jbase >> 1) & 1))) {
-          for (int t = 0; t < n_act; ++t) {
-            issue_qk(t, jbase, L::col_s(t));
-            mma_commit(bar(sh.s_full[t]));
-          }
-          mma_commit(bar(sh.k_empty[jbase & 1]));
-        }
-        for (int j = 0; ok && j < n_blocks; ++j) {
-          const int jg = jbase + j, s = jg & 1;
-          const bool more = j + 1 < n_blocks;
-          for (int t = 0; t < n_act; ++t) {
-            if (!(ok = wait(sh.p_full[t], (jt[t] + j) & 1))) break;
-            if (t == 0 && !(ok = wait(sh.v_full[s], (jg >> 1) & 1))) break;
-            issue_pv(t, jg, j == 0, L::col_s(t));
-            mma_commit(bar(sh.pv_done[t]));
-            if (more) {
-              if (t == 0 && !(ok = wait(sh.k_full[s ^ 1], ((jg + 1) >> 1) & 1))) break;
-              issue_qk(t, jg + 1, L::col_s(t));
-              mma_commit(bar(sh.s_full[t]));
-            }
-          }
-          if (!ok) break;
-          mma_commit(bar(sh.v_empty[s]));
-          if (more) mma_commit(bar(sh.k_empty[s ^ 1]));
-        }
-      }
-      if (!ok && lane == 0) set_abort(sh, p.err);
-    } else {
-      // ----------------------------------------------------- softmax --
-      // Two warpgroups per row tile: warpgroup half h owns key columns
-      // [64 h, 64 h + 64) of every block and output columns [64 h, 64 h + 64).
-      constexpr int kH = L::kHalves;
-      const int t = (warp - 2) / (4 * kH);            // row tile
-      const int h = kH == 2 ? ((warp - 2) >> 2) & 1 : 0;  // column half
-      const int quad = warp & 3;            // TMEM lane quadrant this warp may access
-      const int r_in = quad * 32 + lane;    // row within the tile
-      const int row = t * kRows + r_in;
-      const uint32_t t_lane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
-      const uint32_t o_col = L::col_o(t) + h * (D / kH);
-      const int cnt = NT == 1 ? jbase : jt[t];  // pv_done[t] phases completed before this unit
-      auto tile_sync = [&]() {
-        if (kH == 2) asm volatile("bar.sync %0, %1;" ::"r"(1 + t), "r"(256) : "memory");
-      };
-      if (t < n_act) {
-        // the row's visible keys: prefix below lim_p; own branch's private
-        // keys j <= last, which start at packed page ps
-        const bool valid = row < nrows;
-        const int token = tok0 + row / G;
-        const int bl = valid ? token / m - b_lo : 0;
-        const int lim_p = prefix_limit(row);
-        const int ps = valid ? sh.page_start[bl] : 0;
-        const int last = valid ? sh.blen[bl] - m + (token - (b_lo + bl) * m) : -1;
-        const float sl2 = p.scale_log2;
-        float m_run = NEG_INF, l_half = 0.f;
-        bool ok = true;
-        for (int j = 0; j < n_blocks; ++j) {
-          const int jg = jbase + j;
-          const int si = NT == 1 ? (jg & 1) : t;  // S buffer / barrier index
-          const int ph = NT == 1 ? ((jg >> 1) & 1) : ((jt[t] + j) & 1);
-          const uint32_t s_col = L::col_s(si);
-          // warp-uniform outcome: the tcgen05.ld / st below are warp-collective
-          if (!__all_sync(0xffffffffu, !sh.abort && mbar_wait(bar(sh.s_full[si]), ph))) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const int jb = blk_lo + j;
-          int lo, hi;
-          if (jb < nP) {
-            lo = 0;
-            hi = lim_p - jb * kBlk;
-          } else {
-            const int off = (ps - (jb - nP) * kPagesPerBlock) * kPage;  // column of own key 0
-            lo = max(0, off);
-            hi = min(kBlk, off + last + 1);
-          }
-          const int par = j & 1;
-          auto xchg = [&](float mx) {
-            sh.xmax[h][par][r_in] = mx;
-            tile_sync();
-            return fmaxf(mx, sh.xmax[h ^ 1][par][r_in]);
-          };
-          const float alpha =
-              kH == 2 ? tc::softmax_half_tmem(t_lane + s_col, h, lo, hi, sl2, m_run, l_half, xchg)
-                      : tc::softmax_block_tmem(t_lane + s_col, lo, hi, sl2, m_run, l_half);
-          // Before O may be rescaled, the P V MMA of block j-1 must have
-          // landed.  NT = 2: this tile's S commit was issued after that MMA,
-          // and a commit fires only once every earlier MMA of the issuing
-          // thread has completed, so it has.  NT = 1: P V (j-1) is issued
-          // after Q K^T (j), so a warp that rescales waits for it.  Warps
-          // skip the wait when they do not rescale, yet the parity test stays
-          // exact: Q K^T (j) was issued after P V (j-2), so the S commit
-          // awaited above implies P V (j-2) has completed, and P V (j) needs
-          // this block's P; the barrier is in one of two consecutive phases.
-          // The last block always waits, which gives the epilogue that bound.
-          const bool rescale = __any_sync(0xffffffffu, j > 0 && alpha != 1.f);
-          if (NT == 1 && j > 0 && (rescale || j == n_blocks - 1) &&
-              !__all_sync(0xffffffffu, mbar_wait(bar(sh.pv_done[t]), (cnt + j - 1) & 1))) {
-            ok = false;
-            break;
-          }
-          // Rescale this half's O columns if any row of this warp needs it.
-          if (rescale) {
-            tc_fence_after();
-#pragma unroll
-            for (int c = 0; c < D / kH; c += 32) {
-              uint32_t o[32];
-              tmem_ld32(t_lane + o_col + c, o);
-              tmem_ld_wait();
-#pragma unroll
-              for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-              tmem_st32(t_lane + o_col + c, o);
-            }
-          }
-          tmem_st_wait();
+        const int par = jg & 1;
+        bool xok = true;
+        auto xchg = [&](float mx) {
+          sh.xmax[h][par][r_in] = mx;
           tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(bar(sh.p_full[si]));
-        }
-        if (!ok && lane == 0) set_abort(sh, p.err);
-        // ------------------------------------------------ epilogue --
-        // row sum over both halves (both halves reach this point together:
-        // on a timeout, every wait of the tile's warps gives up)
-        float l_run = l_half;
-        if (kH == 2) {
-          sh.xsum[h][r_in] = l_half;
-          tile_sync();
-          l_run += sh.xsum[h ^ 1][r_in];
-        }
-        // pv_done[t] has completed at least cnt + n_blocks - 1 phases (see
-        // above), so the parity wait for the unit's last block is exact.
-        if (ok && __all_sync(0xffffffffu,
-                             mbar_wait(bar(sh.pv_done[t]), (cnt + n_blocks - 1) & 1))) {
+          publish_seq(&sh.xseq[0][h][quad], jg + 1);
+          xok = await_seq(&sh.xseq[0][h ^ 1][quad], jg + 1, sh);
           tc_fence_after();
-          const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-          const float lse = l_run > 0.f ? (m_run + __log2f(l_run)) * kLn2 : NEG_INF;
+          return fmaxf(mx, sh.xmax[h ^ 1][par][r_in]);
+        };
+        const float alpha =
+            tc::softmax_half_tmem(t_lane + L::col_s(si), h, lo, hi, sl2, m_run, l_half, xchg);
+        if (!(ok = __all_sync(0xffffffffu, xok))) break;
+        // Before O may be rescaled, the P V MMA of block jg-1 must have
+        // landed: a warp that rescales waits for it.  Warps skip the wait
+        // when they do not rescale, yet the parity test stays exact: Q K^T
+        // (jg) was issued after P V (jg-2), so the S commit awaited above
+        // implies P V (jg-2) has completed, and P V (jg) needs this block's
+        // P; the barrier is in one of two consecutive phases.
+        const bool rescale = __any_sync(0xffffffffu, j > 0 && alpha != 1.f);
+        if (rescale) {
+          if (!(ok = wait_bar(sh.pv_done, (jg - 1) & 1))) break;
+          tc_fence_after();
 #pragma unroll
-          for (int c = 0; c < D / kH; c += 32) {
+          for (int c = 0; c < D / 2; c += 32) {
             uint32_t o[32];
             tmem_ld32(t_lane + o_col + c, o);
             tmem_ld_wait();
-            if (!valid) continue;
-            const int dc = h * (D / kH) + c;  // output column
-            if (final_out) {
-              uint4 *dst = reinterpret_cast<uint4 *>(p.out + pair_index(row) * D + dc);
 #pragma unroll
-              for (int e = 0; e < 32; e += 8)
-                dst[e / 8] = make_uint4(
-                    pack_bf16x2(__uint_as_float(o[e]) * inv, __uint_as_float(o[e + 1]) * inv),
-                    pack_bf16x2(__uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv),
-                    pack_bf16x2(__uint_as_float(o[e + 4]) * inv, __uint_as_float(o[e + 5]) * inv),
-                    pack_bf16x2(__uint_as_float(o[e + 6]) * inv, __uint_as_float(o[e + 7]) * inv));
-            } else {
-              float *dst = p.o_part + slot_index(row) * D + dc;
+            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+            tmem_st32(t_lane + o_col + c, o);
+          }
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(sh.p_full[si]));
+      }
+      if (!ok) break;
+      // ---------------------------------------------------- epilogue --
+      // row sum over both halves
+      sh.xsum[h][r_in] = l_half;
+      publish_seq(&sh.xseq[1][h][quad], k + 1);
+      if (!(ok = __all_sync(0xffffffffu, await_seq(&sh.xseq[1][h ^ 1][quad], k + 1, sh)))) break;
+      const float l_run = l_half + sh.xsum[h ^ 1][r_in];
+      if (!(ok = wait_bar(sh.o_full[slot], (k >> 1) & 1))) break;
+      tc_fence_after();
+      const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+      const float lse = l_run > 0.f ? (m_run + __log2f(l_run)) * kLn2 : NEG_INF;
+      const bool final_out = p.S_p == 1;
+      const size_t pair = static_cast<size_t>(token) * p.H_q + g * G + r_in % G;
+      const size_t slot_pair = static_cast<size_t>(split) * p.rows_total * p.H_q + pair;
 #pragma unroll
-              for (int e = 0; e < 32; e += 4)
-                *reinterpret_cast<float4 *>(dst + e) =
-                    make_float4(__uint_as_float(o[e]) * inv, __uint_as_float(o[e + 1]) * inv,
-                                __uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv);
-            }
-          }
-          if (valid && h == 0) {
-            if (final_out) {
-              if (p.lse) p.lse[pair_index(row)] = lse;
-            } else {
-              p.l_part[slot_index(row)] = lse;
-            }
-          }
-          tc_fence_before();  // O is read before the next unit's MMAs overwrite it
-        } else if (ok && lane == 0) {
-          set_abort(sh, p.err);
+      for (int c = 0; c < D / 2; c += 32) {
+        uint32_t o[32];
+        tmem_ld32(t_lane + o_col + c, o);
+        tmem_ld_wait();
+        if (!valid) continue;
+        const int dc = h * (D / 2) + c;  // output column
+        if (final_out) {
+          uint4 *dst = reinterpret_cast<uint4 *>(p.out + pair * D + dc);
+#pragma unroll
+          for (int e = 0; e < 32; e += 8)
+            dst[e / 8] = make_uint4(
+                pack_bf16x2(__uint_as_float(o[e]) * inv, __uint_as_float(o[e + 1]) * inv),
+                pack_bf16x2(__uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv),
+                pack_bf16x2(__uint_as_float(o[e + 4]) * inv, __uint_as_float(o[e + 5]) * inv),
+                pack_bf16x2(__uint_as_float(o[e + 6]) * inv, __uint_as_float(o[e + 7]) * inv));
+        } else {
+          float *dst = p.o_part + slot_pair * D + dc;
+#pragma unroll
+          for (int e = 0; e < 32; e += 4)
+            *reinterpret_cast<float4 *>(dst + e) =
+                make_float4(__uint_as_float(o[e]) * inv, __uint_as_float(o[e + 1]) * inv,
+                            __uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv);
         }
       }
+      if (valid && h == 0) {
+        if (final_out) {
+          if (p.lse) p.lse[pair] = lse;
+        } else {
+          p.l_part[slot_pair] = lse;
+        }
+      }
+      // O slot may be overwritten by unit k + 2 once every warp has read it
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(sh.o_empty[slot]));
+      jbase += nb;
     }
-    // end of unit: every role is done with Q / K / V and with O in TMEM
-    jbase += n_blocks;
-    if (NT == 2) {
-      jt[0] += n_blocks;
-      if (n_act == 2) jt[1] += n_blocks;
-    }
-    ++uidx;
+    if (!ok && lane == 0) set_abort(sh, p.err);
   }
 
   // ------------------------------------------------------------ teardown --
@@ -603,9 +744,10 @@ __global__ void __launch_bounds__(TcLayout<D, NT>::kThreads, 1)
   }
 }
 
-template <int D, int NT>
-cudaError_t launch_tc(const AttnParams &p, const Plan &plan, cudaStream_t s) {
-  using L = TcLayout<D, NT>;
+template <int D>
+cudaError_t launch_tc(const AttnParams &p, cudaStream_t s) {
+  using L = TcLayout<D>;
+  static_assert(L::kDynSmem + sizeof(TcShared) <= 227 * 1024, "shared memory");
   CUtensorMap tq, tk, tv, tkc, tvc;
   cudaError_t e = tc::make_prefix_maps(p, &tq, &tk, &tv);
   if (e == cudaSuccess) e = tc::make_page_map(&tkc, p.k_cache, D, p.H_kv, p.num_pages);
@@ -617,8 +759,7 @@ cudaError_t launch_tc(const AttnParams &p, const Plan &plan, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   const uint64_t bit = 1ull << (dev & 63);
   if (!(configured.load(std::memory_order_acquire) & bit)) {
-    e = cudaFuncSetAttribute(branch_attn_tc_kernel<D, NT>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(branch_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(L::kDynSmem));
     if (e != cudaSuccess) return e;
     configured.fetch_or(bit, std::memory_order_acq_rel);
@@ -630,19 +771,16 @@ cudaError_t launch_tc(const AttnParams &p, const Plan &plan, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     sms[dev & 63] = n;
   }
-  const int n_units = p.n_units;
-  const dim3 grid(static_cast<unsigned>(std::min(n_units, sms[dev & 63])), 1, 1);
-  branch_attn_tc_kernel<D, NT><<<grid, L::kThreads, L::kDynSmem, s>>>(tq, tk, tv, tkc, tvc, p);
+  const dim3 grid(static_cast<unsigned>(std::min(p.n_units, sms[dev & 63])), 1, 1);
+  branch_attn_tc_kernel<D><<<grid, kThreads, L::kDynSmem, s>>>(tq, tk, tv, tkc, tvc, p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_branch_attn_tc(const AttnParams &p, const Plan &plan, cudaStream_t s) {
-  if (plan.tiles_max <= 0) return cudaSuccess;
-  if (plan.tc_tiles == 2)
-    return p.D == 64 ? launch_tc<64, 2>(p, plan, s) : launch_tc<128, 2>(p, plan, s);
-  return p.D == 64 ? launch_tc<64, 1>(p, plan, s) : launch_tc<128, 1>(p, plan, s);
+  if (plan.tiles_max <= 0 || p.n_units <= 0) return cudaSuccess;
+  return p.D == 64 ? launch_tc<64>(p, s) : launch_tc<128>(p, s);
 }
 
 }  // namespace hpd

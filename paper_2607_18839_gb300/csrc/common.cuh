@@ -25,7 +25,6 @@ struct Plan {
   int wr_s;        // warps along rows in the suffix kernel (1, 2, 4)
   int rt_s;        // suffix row tiles per (branch, KV head)
   bool use_tc;     // whole step on tcgen05 (G divides 128) or warp MMA stages
-  int tc_tiles;    // 128-row tiles per tcgen05 prefix CTA (1 or 2)
   size_t off_err;    // uint32 error word
   size_t off_ctr;    // int32 tickets [B][H_kv][rt_s]
   size_t off_opart;  // fp32 [S_p + S_s][rows_total][H_q][D]

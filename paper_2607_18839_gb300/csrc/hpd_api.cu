@@ -55,16 +55,9 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
                                          : a->prefix_tokens;
   pl.use_tc = (a->D == 64 || a->D == 128) && (kTcTileRows % pl.G == 0);
   if (pl.use_tc) {
-    // tcgen05 stage: NT tiles of 128 stacked rows (128 / G tokens each) per
-    // CTA, one CTA per SM.  Two tiles share every K / V load when pages are
-    // big enough to fill them.
-    // Two tiles per CTA share each K / V load, which pays off when a page's
-    // prefix is long (measured: prefix 8,192: 1.5x faster; prefix <= 4,096:
-    // one-tile CTAs, with twice the units and a split softmax, are as fast
-    // or faster).
-    const long long stacked = static_cast<long long>(a->B) * a->m * pl.G;
-    pl.tc_tiles = (stacked >= 2LL * kTcTileRows * a->n_docs && maxP >= 48 * 128) ? 2 : 1;
-    const int tile_tokens = pl.tc_tiles * (kTcTileRows / pl.G);
+    // tcgen05 kernel: units of 128 stacked rows (128 / G tokens) of one
+    // page and KV head, one CTA per SM taking units in turn.
+    const int tile_tokens = kTcTileRows / pl.G;
     const int tiles = ceil_div(static_cast<long long>(a->B) * a->m, tile_tokens);
     pl.tiles_max = tiles + a->n_docs;
     // Key splits: minimise the estimated time of the step, i.e. waves of
@@ -74,11 +67,11 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
     // (guessed at a quarter of the page-table width per branch).
     const long long ctas = static_cast<long long>(std::max(tiles, 1)) * a->H_kv;
     const int branches_per_cta =
-        std::max(1, (pl.tc_tiles * kTcTileRows) / std::max(1, a->m * pl.G));
+        std::max(1, kTcTileRows / std::max(1, a->m * pl.G));
     const int nb = std::max(1, ceil_div(maxP, 128)) +
                    ceil_div(static_cast<long long>(branches_per_cta) *
                                 std::max(1, a->max_pages_per_branch / 4), 8);
-    const double block_us = 1.3 * pl.tc_tiles;  // one 128-key block, measured order
+    const double block_us = 0.7;  // one 128-key block, measured order
     const double partial_bytes =
         static_cast<double>(a->B) * a->m * a->H_q * (a->D + 1) * sizeof(float);
     int best = 1;

@@ -45,14 +45,24 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Wait for the completion of the phase with parity `parity`; false on timeout.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-  if (mbar_try_wait(bar, parity)) return true;
+// Slow path of mbar_wait: poll until the phase completes (true), the time
+// limit passes or *abort becomes non-zero (false).  Kept out of line so that
+// the clock read cannot be hoisted into the fast path.
+__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, const int *abort) {
   const uint64_t t0 = globaltimer();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 0 && globaltimer() - t0 > kWaitLimitNs) return false;
+    if ((i & 255u) == 0) {
+      if (abort && *reinterpret_cast<const volatile int *>(abort)) return false;
+      if (globaltimer() - t0 > kWaitLimitNs) return false;
+    }
   }
+}
+// Wait for the completion of the phase with parity `parity`; false on
+// timeout (or when *abort, if given, becomes non-zero while waiting).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
+                                          const int *abort = nullptr) {
+  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, abort);
 }
 
 // ----------------------------------------------------------------- TMA --

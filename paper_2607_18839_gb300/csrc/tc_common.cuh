@@ -1,6 +1,6 @@
-// tc_common.cuh -- pieces shared by the tcgen05 shared-prefix kernels:
-// locating a CTA's row tile, one 128-key block of a row's online softmax,
-// and TMA tensor-map encoding on the host.
+// tc_common.cuh -- pieces of the tcgen05 branch-attention kernel: half of a
+// 128-key block of a row's online softmax, and TMA tensor-map encoding on
+// the host.
 #pragma once
 
 #include <cudaTypedefs.h>
@@ -23,170 +23,6 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 constexpr int kRows = 128;  // stacked query rows of one tile (MMA M)
 constexpr int kBlk = 128;   // keys per block (MMA N of S = Q K^T)
 constexpr float kRescaleLog2 = 8.0f;  // tolerate a stale row max up to 2^8
-
-// Warp 0 finds the page owning row-tile `tile` of KV head blockIdx.y, where
-// page d has ceil(#branches(d) * m / tile_tokens) tiles, and writes
-// {d, tile index within d, first branch, end branch} to info (-1: no tile).
-__device__ __forceinline__ void locate_tile(const AttnParams &p, int tile, int tile_tokens,
-                                            int *info) {
-  const int lane = threadIdx.x & 31;
-  int base = 0;
-  for (int d0 = 0; d0 < p.n_docs; d0 += 32) {
-    const int d = d0 + lane;
-    int tiles = 0, b0 = 0, b1 = 0;
-    if (d < p.n_docs) {
-      b0 = min(max(p.branch_cu[d], 0), p.B);
-      b1 = min(max(p.branch_cu[d + 1], 0), p.B);
-      if (b1 < b0) {
-        flag_error(p.err, HPD_DEVERR_BRANCH_CU);
-        b1 = b0;
-      }
-      tiles = ceil_div_i((b1 - b0) * p.m, tile_tokens);
-    }
-    int incl = tiles;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int v = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += v;
-    }
-    const int excl = incl - tiles;
-    if (tiles > 0 && tile >= base + excl && tile < base + incl) {
-      info[0] = d;
-      info[1] = tile - base - excl;
-      info[2] = b0;
-      info[3] = b1;
-    }
-    base += __shfl_sync(0xffffffffu, incl, 31);
-    if (base > tile) break;
-  }
-}
-
-// One 128-key block of a row's online softmax (base 2, scaled scores).
-// s_addr is this thread's lane at the block's fp32 scores in TMEM; only
-// columns [lo, hi) are visible to the row.  The bf16 probabilities, relative
-// to the (possibly stale) running max, are written back over the scores as
-// 64 packed columns.  Updates m_run / l_run and returns the factor by which
-// the row's accumulated output must be rescaled (1 if unchanged).
-// Warp-collective (tcgen05.ld / st): all 32 lanes of the warp must call it
-// together.  Three paths, chosen per warp:
-//   no row of the warp sees the block   zeros, no loads
-//   every row sees all 128 columns      unrolled over the 128 scores held
-//                                       in registers
-//   otherwise                           a compact loop over 32-column chunks
-//                                       that reloads them from TMEM
-__device__ __forceinline__ float softmax_block_tmem(uint32_t s_addr, int lo, int hi, float sl2,
-                                                    float &m_run, float &l_run) {
-  using namespace sm100;
-  const float NEG_INF = -__int_as_float(0x7f800000);
-  lo = max(lo, 0);
-  hi = min(hi, kBlk);
-  if (__all_sync(0xffffffffu, hi <= lo)) {
-    uint32_t z[16];
-#pragma unroll
-    for (int c = 0; c < 16; ++c) z[c] = 0u;
-#pragma unroll
-    for (int ch = 0; ch < kBlk / 32; ++ch) tmem_st16(s_addr + ch * 16, z);
-    return 1.f;
-  }
-  float m_new, base, alpha, sum;
-  if (__all_sync(0xffffffffu, lo == 0 && hi == kBlk)) {
-    uint32_t v[kBlk];
-#pragma unroll
-    for (int ch = 0; ch < kBlk / 32; ++ch) tmem_ld32(s_addr + ch * 32, v + ch * 32);
-    tmem_ld_wait();
-    // row max with three-input max over 8 independent chains; on the raw
-    // scores when the scale is positive (it keeps the order), else scaled
-    float mx8[8];
-#pragma unroll
-    for (int a = 0; a < 8; ++a) mx8[a] = NEG_INF;
-    if (sl2 > 0.f) {
-#pragma unroll
-      for (int c = 0; c < kBlk; c += 16)
-#pragma unroll
-        for (int a = 0; a < 8; ++a)
-          mx8[a] = fmax3(mx8[a], __uint_as_float(v[c + 2 * a]), __uint_as_float(v[c + 2 * a + 1]));
-    } else {
-#pragma unroll
-      for (int c = 0; c < kBlk; c += 16)
-#pragma unroll
-        for (int a = 0; a < 8; ++a)
-          mx8[a] = fmax3(mx8[a], __uint_as_float(v[c + 2 * a]) * sl2,
-                         __uint_as_float(v[c + 2 * a + 1]) * sl2);
-    }
-    float mx = fmax3(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(mx8[3], mx8[4], mx8[5]),
-                     fmaxf(mx8[6], mx8[7]));
-    if (sl2 > 0.f) mx *= sl2;
-    m_new = mx > m_run + kRescaleLog2 ? mx : m_run;
-    base = m_new == NEG_INF ? 0.f : m_new;
-    alpha = m_new == m_run ? 1.f : fast_exp2(m_run - base);
-    // exponent arguments and running sums two lanes at a time (fp32x2 FMA / add)
-    const float2 sl2x2 = make_float2(sl2, sl2), nbase2 = make_float2(-base, -base);
-    float2 sum4[4];
-#pragma unroll
-    for (int a = 0; a < 4; ++a) sum4[a] = make_float2(0.f, 0.f);
-#pragma unroll
-    for (int ch = 0; ch < kBlk / 32; ++ch) {
-      uint32_t pk[16];
-#pragma unroll
-      for (int c = 0; c < 32; c += 2) {
-        const float2 x = make_float2(__uint_as_float(v[ch * 32 + c]),
-                                     __uint_as_float(v[ch * 32 + c + 1]));
-        const float2 arg = __ffma2_rn(x, sl2x2, nbase2);
-        const float2 e = make_float2(fast_exp2(arg.x), fast_exp2(arg.y));
-        sum4[(c >> 1) & 3] = __fadd2_rn(sum4[(c >> 1) & 3], e);
-        pk[c / 2] = pack_bf16x2(e.x, e.y);
-      }
-      tmem_st16(s_addr + ch * 16, pk);
-    }
-    const float2 s01 = __fadd2_rn(sum4[0], sum4[1]), s23 = __fadd2_rn(sum4[2], sum4[3]);
-    const float2 s03 = __fadd2_rn(s01, s23);
-    sum = s03.x + s03.y;
-  } else {
-    // pass 1: max over the visible columns, chunk by chunk
-    float mx = NEG_INF;
-#pragma unroll 1
-    for (int ch = 0; ch < kBlk / 32; ++ch) {
-      uint32_t v[32];
-      tmem_ld32(s_addr + ch * 32, v);
-      tmem_ld_wait();
-      float mx4[4] = {NEG_INF, NEG_INF, NEG_INF, NEG_INF};
-#pragma unroll
-      for (int c = 0; c < 32; ++c) {
-        const int col = ch * 32 + c;
-        mx4[c & 3] = fmaxf(mx4[c & 3], col >= lo && col < hi ? __uint_as_float(v[c]) * sl2 : NEG_INF);
-      }
-      mx = fmaxf(mx, fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3])));
-    }
-    m_new = mx > m_run + kRescaleLog2 ? mx : m_run;
-    base = m_new == NEG_INF ? 0.f : m_new;
-    alpha = m_new == m_run ? 1.f : fast_exp2(m_run - base);
-    // pass 2: probabilities; P chunk ch lands in columns [16 ch, 16 ch + 16),
-    // below the next chunk still to be read (32 ch + 32)
-    sum = 0.f;
-#pragma unroll 1
-    for (int ch = 0; ch < kBlk / 32; ++ch) {
-      uint32_t v[32], pk[16];
-      tmem_ld32(s_addr + ch * 32, v);
-      tmem_ld_wait();
-      float s4[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int c = 0; c < 32; c += 2) {
-        const int col = ch * 32 + c;
-        const float e0 = col >= lo && col < hi
-                             ? fast_exp2(fmaf(__uint_as_float(v[c]), sl2, -base)) : 0.f;
-        const float e1 = col + 1 >= lo && col + 1 < hi
-                             ? fast_exp2(fmaf(__uint_as_float(v[c + 1]), sl2, -base)) : 0.f;
-        s4[(c >> 1) & 3] += e0 + e1;
-        pk[c / 2] = pack_bf16x2(e0, e1);
-      }
-      tmem_st16(s_addr + ch * 16, pk);
-      sum += (s4[0] + s4[1]) + (s4[2] + s4[3]);
-    }
-  }
-  l_run = l_run * alpha + sum;
-  m_run = m_new;
-  return alpha;
-}
 
 // Half of one 128-key block of a row's online softmax: this thread owns the
 // 64 columns [64 h, 64 h + 64) of its row; the thread of the other half (the
