@@ -45,17 +45,29 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Slow path of mbar_wait: poll until the phase completes (true), the time
-// limit passes or *abort becomes non-zero (false).  Kept out of line so that
-// the clock read cannot be hoisted into the fast path.
+// try_wait that lets the thread sleep until the phase completes, for at most
+// about `ns` nanoseconds, so that waiting warps leave the issue slots of
+// their SM sub-partition to the warps that compute.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(ns)
+      : "memory");
+  return ok != 0;
+}
+// Slow path of mbar_wait: sleep-wait until the phase completes (true), the
+// time limit passes or *abort becomes non-zero (false).  Kept out of line so
+// that the clock read cannot be hoisted into the fast path.
 __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, const int *abort) {
   const uint64_t t0 = globaltimer();
-  for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 0) {
-      if (abort && *reinterpret_cast<const volatile int *>(abort)) return false;
-      if (globaltimer() - t0 > kWaitLimitNs) return false;
-    }
+  for (;;) {
+    if (mbar_try_wait_sleep(bar, parity, 100000u)) return true;
+    if (abort && *reinterpret_cast<const volatile int *>(abort)) return false;
+    if (globaltimer() - t0 > kWaitLimitNs) return false;
   }
 }
 // Wait for the completion of the phase with parity `parity`; false on
