@@ -27,23 +27,27 @@
 //   warp 10     scheduler: takes the next unit and prepares its metadata
 //               (page, rows, private lengths, fork limits, packed page ids)
 //               in one of two shared-memory slots while the other is in use.
-//   warps 0, 11 TMA producers: warp 0 the unit's Q tile into one of two Q
-//               slots and its K blocks, warp 11 its V blocks, each into a
-//               two-stage ring (128-byte swizzle); a K stage is refilled as
-//               soon as its Q K^T is done, whatever the V ring waits for.
+//   warps 0, 11 TMA producers: warp 0 the unit's K blocks, warp 11 its V
+//               blocks, each into a three-stage ring (128-byte swizzle); a K
+//               stage is refilled as soon as its Q K^T is done, whatever the
+//               V ring waits for.
 //   warp 1      TMEM owner and MMA issuer; one global sequence of blocks
 //               across units, in the order QK(b), PV(b-1):
-//                 S = Q K^T   -> TMEM (fp32, double buffered by block)
-//                 O += P V    P read from TMEM (bf16, written over S); O in
-//                             TMEM, double buffered by unit so a unit's
-//                             epilogue overlaps the next unit's MMAs.
+//                 S = Q K^T   Q read from TMEM, K from shared memory; S into
+//                             TMEM (fp32, double buffered by block)
+//                 O += P V    P read from TMEM (bf16, written over S), V from
+//                             shared memory; O accumulated in TMEM
+//               With both A operands in TMEM, shared memory serves only K,
+//               V and their TMA writes (its bandwidth is the scarce port).
 //   warps 2..9  softmax: two warpgroups, each owning half of every block's
 //               128 key columns and half of O's columns; thread t of warp w
 //               owns TMEM lane 32*(w%4)+t, i.e. one query row.  The two
 //               halves of a row exchange their partial max through shared
 //               memory.  O is rescaled in TMEM only when a row's running
 //               max grows by more than 2^8; the stale max stays exact after
-//               the final normalisation.
+//               the final normalisation.  They also copy each unit's Q rows
+//               from global memory into TMEM (double buffered by unit), the
+//               next unit's before the current unit's epilogue.
 // One split: the unit writes the final bf16 output and lse.  Several splits:
 // it writes its normalised fp32 partial and lse for merge.cu.
 // All waits are bounded; a timeout sets HPD_DEVERR_TIMEOUT, every role
@@ -72,7 +76,7 @@ constexpr int kVWarp = kSchedWarp + 1;
 constexpr int kThreads = 32 * (kVWarp + 1);
 // consumers of a metadata slot: two producers, MMA issuer, softmax warps
 constexpr uint32_t kMetaConsumers = 3 + kSoftmaxWarps;
-constexpr int kMaxRing = 3;  // largest Q / K / V ring
+constexpr int kMaxRing = 3;  // largest K / V ring
 
 // Metadata of one unit, written by the scheduler warp.
 struct UnitMeta {
@@ -99,26 +103,27 @@ struct TcLayout {
   static constexpr int kChunks = D / 64;                // 64-column (128-byte) boxes
   static constexpr uint32_t kChunkBytes = kRows * 128;  // 128 rows x 128 bytes
   static constexpr uint32_t kTileBytes = kChunks * kChunkBytes;
-  static constexpr int kQSlots = 2, kKStages = 2, kVStages = 2;
-  static constexpr uint32_t kQ = 0;
-  static constexpr uint32_t kK = kQSlots * kTileBytes;
+  static constexpr int kKStages = 3, kVStages = 3;
+  static constexpr uint32_t kK = 0;
   static constexpr uint32_t kV = kK + kKStages * kTileBytes;
   static constexpr uint32_t kMeta = kV + kVStages * kTileBytes;  // 2 UnitMeta slots
   static constexpr uint32_t kBytes = kMeta + 2 * sizeof(UnitMeta);
   static constexpr uint32_t kDynSmem = kBytes + 1024;   // slack to align to 1024
-  // TMEM columns: S of block buffer i at col_s(i), O of unit slot o at col_o(o)
+  // TMEM columns: S of block buffer i at col_s(i), O at kColO, the Q rows of
+  // unit slot u at col_q(u) (D / 2 columns: two bf16 per column)
+  static constexpr uint32_t kColO = 256;
   static __device__ __forceinline__ uint32_t col_s(int i) { return i ? 128u : 0u; }
-  static __device__ __forceinline__ uint32_t col_o(int o) { return o ? 384u : 256u; }
+  static __device__ __forceinline__ uint32_t col_q(int u) { return u ? 448u : 384u; }
 };
 
 struct __align__(8) TcShared {
   uint64_t meta_full[2], meta_empty[2];
-  uint64_t q_full[kMaxRing], q_empty[kMaxRing];
+  uint64_t q_full[2], q_empty[2];  // Q rows in TMEM, per unit slot
   uint64_t k_full[kMaxRing], v_full[kMaxRing];
   uint64_t k_empty[kMaxRing], v_empty[kMaxRing];
   uint64_t s_full[2], p_full[2];  // per S buffer
   uint64_t pv_done;
-  uint64_t o_full[2], o_empty[2];  // per O slot
+  uint64_t o_full, o_empty;
   uint64_t mma_done;
   uint32_t tmem_base;
   int abort;
@@ -169,8 +174,7 @@ __device__ __forceinline__ bool await_seq(const int *flag, int seq, const TcShar
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
-    branch_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
-                          const __grid_constant__ CUtensorMap tm_k,
+    branch_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k,
                           const __grid_constant__ CUtensorMap tm_v,
                           const __grid_constant__ CUtensorMap tm_kc,
                           const __grid_constant__ CUtensorMap tm_vc, const AttnParams p) {
@@ -194,8 +198,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) {
     sh.abort = 0;
     for (int s = 0; s < kMaxRing; ++s) {
-      mbar_init(bar(sh.q_full[s]), 1);
-      mbar_init(bar(sh.q_empty[s]), 1);
       mbar_init(bar(sh.k_full[s]), 1);
       mbar_init(bar(sh.v_full[s]), 1);
       mbar_init(bar(sh.k_empty[s]), 1);
@@ -206,10 +208,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar(sh.meta_empty[s]), kMetaConsumers);
       mbar_init(bar(sh.s_full[s]), 1);
       mbar_init(bar(sh.p_full[s]), kSoftmaxWarps);
-      mbar_init(bar(sh.o_full[s]), 1);
-      mbar_init(bar(sh.o_empty[s]), kSoftmaxWarps);
+      mbar_init(bar(sh.q_full[s]), kSoftmaxWarps);
+      mbar_init(bar(sh.q_empty[s]), 1);
     }
     mbar_init(bar(sh.pv_done), 1);
+    mbar_init(bar(sh.o_full), 1);
+    mbar_init(bar(sh.o_empty), kSoftmaxWarps);
     mbar_init(bar(sh.mma_done), 1);
     fence_mbar_init();
   }
@@ -400,14 +404,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     // lane issues each copy.  Warp 0: Q and K; warp kVWarp: V.
     const bool is_k = warp == 0;
     if (lane == 0) {
-      prefetch_tmap(&tm_q);
       prefetch_tmap(&tm_k);
       prefetch_tmap(&tm_v);
       prefetch_tmap(&tm_kc);
       prefetch_tmap(&tm_vc);
     }
     __syncwarp();
-    int jbase = 0, issued_k = 0, issued_v = 0, issued_q = 0;
+    int jbase = 0, issued_k = 0, issued_v = 0;
     bool ok = true;
     for (int k = 0; ok; ++k) {
       const int slot = k & 1;
@@ -416,19 +419,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!M.valid) break;
       const int g = M.g, nP = M.nP, pc0 = M.pc0, blk_lo = M.blk_lo, nb = M.n_blocks;
       const int P_s = M.page_start[M.nbc];
-      // Q tile into slot k % kQSlots, once the Q K^T MMAs of the unit that
-      // used it last are done
-      if (is_k) {
-        const int qs = k % L::kQSlots;
-        if (k >= L::kQSlots &&
-            !(ok = wait_bar(sh.q_empty[qs], ((k / L::kQSlots) - 1) & 1)))
-          break;
-        mbar_arrive_expect_tx_elect(bar(sh.q_full[qs]), L::kTileBytes);
-        for (int c = 0; c < L::kChunks; ++c)
-          tma_load_3d_elect(sbase + L::kQ + qs * L::kTileBytes + c * L::kChunkBytes, &tm_q,
-                            bar(sh.q_full[qs]), c * 64, g * G, M.tok0);
-        issued_q = k + 1;
-      }
       // page id of packed suffix page gp (past the shared-memory table: looked
       // up again; an id out of range was flagged by the scheduler)
       auto page_of = [&](int gp) -> int {
@@ -492,8 +482,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!ok && lane == 0) set_abort(sh, p.err);
     // Do not exit while a copy into this CTA's shared memory is in flight:
     // wait for the most recent phase of every barrier a copy may complete.
-    for (int q = max(0, issued_q - L::kQSlots); q < issued_q; ++q)
-      mbar_wait(bar(sh.q_full[q % L::kQSlots]), (q / L::kQSlots) & 1);
     for (int jg = max(0, issued_k - L::kKStages); jg < issued_k; ++jg)
       mbar_wait(bar(sh.k_full[jg % L::kKStages]), (jg / L::kKStages) & 1);
     for (int jg = max(0, issued_v - L::kVStages); jg < issued_v; ++jg)
@@ -507,28 +495,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Shared-memory descriptors: a slot / stage / k-step offset only adds
     // (offset >> 4) to the start-address field (bits 0-13), which cannot
     // carry: every address stays below 256 KB.
-    const uint64_t dq0 = smem_desc_sw128(sbase + L::kQ, 16, 1024);
     const uint64_t dk0 = smem_desc_sw128(sbase + L::kK, 16, 1024);
-    // S[col] = Q (slot qs) K^T of global block jg
+    // S[col] = Q (TMEM slot qs) K^T of global block jg: A from TMEM, 16
+    // dimensions (8 columns) per MMA; B = K, K-major in shared memory
     auto issue_qk = [&](int qs, int jg, uint32_t col) {
-      const uint64_t qd = dq0 + ((qs * L::kTileBytes) >> 4);
       const uint64_t kd = dk0 + (((jg % L::kKStages) * L::kTileBytes) >> 4);
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t off = ((kk >> 2) * L::kChunkBytes + (kk & 3) * 32) >> 4;
-        mma_ss(tmem + col, qd + off, kd + off, idesc_qk, kk > 0);
+        mma_ts(tmem + col, tmem + L::col_q(qs) + kk * 8, kd + off, idesc_qk, kk > 0);
       }
     };
-    // O (slot os) (+)= P V of global block jg, P in TMEM at column pcol: one
+    // O (+)= P V of global block jg, P in TMEM at column pcol: one
     // N = D MMA per 16 keys.  V is MN-major (D contiguous): 64-column swizzle
     // atoms kChunkBytes apart along N (leading byte offset), 8-key groups
     // 1024 bytes apart along K (stride byte offset).
     const uint64_t dv0 = smem_desc_sw128(sbase + L::kV, L::kChunkBytes, 1024);
-    auto issue_pv = [&](int os, int jg, bool first, uint32_t pcol) {
+    auto issue_pv = [&](int jg, bool first, uint32_t pcol) {
       const uint64_t vd = dv0 + (((jg % L::kVStages) * L::kTileBytes) >> 4);
 #pragma unroll
       for (int kk = 0; kk < kBlk / 16; ++kk)
-        mma_ts(tmem + L::col_o(os), tmem + pcol + kk * 8, vd + ((kk * 16 * 128) >> 4), idesc_pv,
+        mma_ts(tmem + L::kColO, tmem + pcol + kk * 8, vd + ((kk * 16 * 128) >> 4), idesc_pv,
                (!first || kk > 0) ? 1u : 0u);
     };
     auto wait = [&](uint64_t &b, int parity) {
@@ -545,15 +532,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     Pending pend{0, 0, false, false};
     bool has_pend = false;
     auto do_pv = [&](const Pending &x) -> bool {
-      const int s = x.jg & 1, os = x.unit & 1, sv = x.jg % L::kVStages;
+      const int s = x.jg & 1, sv = x.jg % L::kVStages;
       if (!wait(sh.p_full[s], (x.jg >> 1) & 1) || !wait(sh.v_full[sv], (x.jg / L::kVStages) & 1))
         return false;
-      // O slot os last held unit x.unit - 2, whose epilogue must have read it
-      if (x.first && x.unit >= 2 && !wait(sh.o_empty[os], ((x.unit >> 1) - 1) & 1)) return false;
-      issue_pv(os, x.jg, x.first, L::col_s(s));
+      // O last held unit x.unit - 1, whose epilogue must have read it
+      if (x.first && x.unit >= 1 && !wait(sh.o_empty, (x.unit - 1) & 1)) return false;
+      issue_pv(x.jg, x.first, L::col_s(s));
       mma_commit(bar(sh.pv_done));
       mma_commit(bar(sh.v_empty[sv]));
-      if (x.last) mma_commit(bar(sh.o_full[os]));
+      if (x.last) mma_commit(bar(sh.o_full));
       return true;
     };
     int jbase = 0;
@@ -566,8 +553,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (!valid) break;
       if (lane == 0) mbar_arrive(bar(sh.meta_empty[slot]));
-      const int qs = k % L::kQSlots;
-      if (!(ok = wait(sh.q_full[qs], (k / L::kQSlots) & 1))) break;
+      const int qs = k & 1;
+      if (!(ok = wait(sh.q_full[qs], (k >> 1) & 1))) break;
       for (int j = 0; j < nb; ++j) {
         const int jg = jbase + j, s = jg & 1, sk = jg % L::kKStages;
         if (!(ok = wait(sh.k_full[sk], (jg / L::kKStages) & 1))) break;
@@ -592,42 +579,88 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r_in = quad * 32 + lane;    // row within the tile
     const uint32_t t_lane = tmem + (static_cast<uint32_t>(quad * 32) << 16);
     const float sl2 = p.scale_log2;
-    int jbase = 0;
-    bool ok = true;
-    for (int k = 0; ok; ++k) {
+    // This thread's row of a unit: where it reads Q and writes the output,
+    // and its visible keys (prefix below lim_p; own branch's private keys
+    // j <= last, which start at packed page ps).
+    struct Row {
+      bool unit;  // false: no unit left
+      bool valid;
+      int g, split, nb, blk_lo, nP, lim_p, ps, last;
+      size_t pair;
+    };
+    // Reads unit k's metadata (slot k & 1), releases the slot, and copies the
+    // row's half of Q (D / 2 dimensions) into TMEM slot k & 1 once unit k - 2's
+    // Q K^T MMAs are done with it; false on timeout / abort.
+    auto begin_unit = [&](int k, Row &R) -> bool {
       const int slot = k & 1;
-      if (!(ok = wait_bar(sh.meta_full[slot], (k >> 1) & 1))) break;
+      if (!wait_bar(sh.meta_full[slot], (k >> 1) & 1)) return false;
       const UnitMeta &M = meta[slot];
-      if (!M.valid) break;
-      const int g = M.g, split = M.split, tok0 = M.tok0, nb = M.n_blocks;
-      const int blk_lo = M.blk_lo, nP = M.nP;
-      // the row's visible keys: prefix below lim_p; own branch's private
-      // keys j <= last, which start at packed page ps
-      const bool valid = r_in < M.nrows;
-      const int token = tok0 + r_in / G;
-      const int bl = valid ? token / m - M.b_lo : 0;
-      const int lim_p = valid ? M.fork[bl] : 0;
-      const int ps = valid ? M.page_start[bl] : 0;
-      const int last = valid ? M.blen[bl] - m + (token - (M.b_lo + bl) * m) : -1;
+      R.unit = M.valid != 0;
+      if (R.unit) {
+        R.g = M.g;
+        R.split = M.split;
+        R.nb = M.n_blocks;
+        R.blk_lo = M.blk_lo;
+        R.nP = M.nP;
+        R.valid = r_in < M.nrows;
+        const int token = M.tok0 + r_in / G;
+        const int bl = R.valid ? token / m - M.b_lo : 0;
+        R.lim_p = R.valid ? M.fork[bl] : 0;
+        R.ps = R.valid ? M.page_start[bl] : 0;
+        R.last = R.valid ? M.blen[bl] - m + (token - (M.b_lo + bl) * m) : -1;
+        R.pair = static_cast<size_t>(token) * p.H_q + R.g * G + r_in % G;
+      }
       __syncwarp();
+      if (!R.unit) return true;
       if (lane == 0) mbar_arrive(bar(sh.meta_empty[slot]));
-      const uint32_t o_col = L::col_o(slot) + h * (D / 2);
+      uint32_t w[D / 4];
+      if (R.valid) {
+        const uint4 *src = reinterpret_cast<const uint4 *>(p.q + R.pair * D + h * (D / 2));
+#pragma unroll
+        for (int i = 0; i < D / 16; ++i) {
+          const uint4 x = __ldg(src + i);
+          w[4 * i] = x.x;
+          w[4 * i + 1] = x.y;
+          w[4 * i + 2] = x.z;
+          w[4 * i + 3] = x.w;
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < D / 4; ++i) w[i] = 0u;
+      }
+      if (k >= 2 && !wait_bar(sh.q_empty[slot], ((k >> 1) - 1) & 1)) return false;
+      tc_fence_after();
+      if constexpr (D == 128)
+        tmem_st32(t_lane + L::col_q(slot) + h * (D / 4), w);
+      else
+        tmem_st16(t_lane + L::col_q(slot) + h * (D / 4), w);
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(sh.q_full[slot]));
+      return true;
+    };
+    const uint32_t o_col = L::kColO + h * (D / 2);
+    int jbase = 0;
+    Row cur{}, nxt{};
+    bool ok = begin_unit(0, cur);
+    for (int k = 0; ok && cur.unit; ++k) {
       float m_run = NEG_INF, l_half = 0.f;
-      for (int j = 0; j < nb; ++j) {
+      for (int j = 0; j < cur.nb; ++j) {
         const int jg = jbase + j;
         const int si = jg & 1;
         // warp-uniform outcome: the tcgen05.ld / st below are warp-collective
         if (!(ok = wait_bar(sh.s_full[si], (jg >> 1) & 1))) break;
         tc_fence_after();
-        const int jb = blk_lo + j;
+        const int jb = cur.blk_lo + j;
         int lo, hi;
-        if (jb < nP) {
+        if (jb < cur.nP) {
           lo = 0;
-          hi = lim_p - jb * kBlk;
+          hi = cur.lim_p - jb * kBlk;
         } else {
-          const int off = (ps - (jb - nP) * kPagesPerBlock) * kPage;  // column of own key 0
+          const int off = (cur.ps - (jb - cur.nP) * kPagesPerBlock) * kPage;  // column of own key 0
           lo = max(0, off);
-          hi = min(kBlk, off + last + 1);
+          hi = min(kBlk, off + cur.last + 1);
         }
         const int par = jg & 1;
         bool xok = true;
@@ -668,28 +701,30 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(bar(sh.p_full[si]));
       }
       if (!ok) break;
+      // the next unit's Q goes to TMEM before this unit's epilogue, so that
+      // its first Q K^T MMAs run meanwhile
+      if (!(ok = begin_unit(k + 1, nxt))) break;
       // ---------------------------------------------------- epilogue --
       // row sum over both halves
       sh.xsum[h][r_in] = l_half;
       publish_seq(&sh.xseq[1][h][quad], k + 1);
       if (!(ok = __all_sync(0xffffffffu, await_seq(&sh.xseq[1][h ^ 1][quad], k + 1, sh)))) break;
       const float l_run = l_half + sh.xsum[h ^ 1][r_in];
-      if (!(ok = wait_bar(sh.o_full[slot], (k >> 1) & 1))) break;
+      if (!(ok = wait_bar(sh.o_full, k & 1))) break;
       tc_fence_after();
       const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
       const float lse = l_run > 0.f ? (m_run + __log2f(l_run)) * kLn2 : NEG_INF;
       const bool final_out = p.S_p == 1;
-      const size_t pair = static_cast<size_t>(token) * p.H_q + g * G + r_in % G;
-      const size_t slot_pair = static_cast<size_t>(split) * p.rows_total * p.H_q + pair;
+      const size_t slot_pair = static_cast<size_t>(cur.split) * p.rows_total * p.H_q + cur.pair;
 #pragma unroll
       for (int c = 0; c < D / 2; c += 32) {
         uint32_t o[32];
         tmem_ld32(t_lane + o_col + c, o);
         tmem_ld_wait();
-        if (!valid) continue;
+        if (!cur.valid) continue;
         const int dc = h * (D / 2) + c;  // output column
         if (final_out) {
-          uint4 *dst = reinterpret_cast<uint4 *>(p.out + pair * D + dc);
+          uint4 *dst = reinterpret_cast<uint4 *>(p.out + cur.pair * D + dc);
 #pragma unroll
           for (int e = 0; e < 32; e += 8)
             dst[e / 8] = make_uint4(
@@ -706,18 +741,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                             __uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv);
         }
       }
-      if (valid && h == 0) {
+      if (cur.valid && h == 0) {
         if (final_out) {
-          if (p.lse) p.lse[pair] = lse;
+          if (p.lse) p.lse[cur.pair] = lse;
         } else {
           p.l_part[slot_pair] = lse;
         }
       }
-      // O slot may be overwritten by unit k + 2 once every warp has read it
+      // O may be overwritten by the next unit once every warp has read it
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(bar(sh.o_empty[slot]));
-      jbase += nb;
+      if (lane == 0) mbar_arrive(bar(sh.o_empty));
+      jbase += cur.nb;
+      cur = nxt;
     }
     if (!ok && lane == 0) set_abort(sh, p.err);
   }
@@ -748,8 +784,8 @@ template <int D>
 cudaError_t launch_tc(const AttnParams &p, cudaStream_t s) {
   using L = TcLayout<D>;
   static_assert(L::kDynSmem + sizeof(TcShared) <= 227 * 1024, "shared memory");
-  CUtensorMap tq, tk, tv, tkc, tvc;
-  cudaError_t e = tc::make_prefix_maps(p, &tq, &tk, &tv);
+  CUtensorMap tk, tv, tkc, tvc;
+  cudaError_t e = tc::make_prefix_maps(p, &tk, &tv);
   if (e == cudaSuccess) e = tc::make_page_map(&tkc, p.k_cache, D, p.H_kv, p.num_pages);
   if (e == cudaSuccess) e = tc::make_page_map(&tvc, p.v_cache, D, p.H_kv, p.num_pages);
   if (e != cudaSuccess) return e;
@@ -772,7 +808,7 @@ cudaError_t launch_tc(const AttnParams &p, cudaStream_t s) {
     sms[dev & 63] = n;
   }
   const dim3 grid(static_cast<unsigned>(std::min(p.n_units, sms[dev & 63])), 1, 1);
-  branch_attn_tc_kernel<D><<<grid, kThreads, L::kDynSmem, s>>>(tq, tk, tv, tkc, tvc, p);
+  branch_attn_tc_kernel<D><<<grid, kThreads, L::kDynSmem, s>>>(tk, tv, tkc, tvc, p);
   return cudaGetLastError();
 }
 

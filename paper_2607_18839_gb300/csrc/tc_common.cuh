@@ -186,15 +186,14 @@ inline cudaError_t make_page_map(CUtensorMap *map, const void *base, int D, int 
 
 // Maps of Q (box: 64 columns x G heads x 128/G tokens = one 128-row tile)
 // and of the prefix K / V (box: 64 columns x 1 head x 128 keys).
-inline cudaError_t make_prefix_maps(const AttnParams &p, CUtensorMap *tq, CUtensorMap *tk,
-                                    CUtensorMap *tv) {
-  const int D = p.D, G = p.G;
-  cudaError_t e = make_map(tq, p.q, D, p.H_q, static_cast<uint64_t>(p.rows_total), 64, G,
-                           kRows / G);
-  if (e != cudaSuccess) return e;
+// K and V maps of the contiguous prefix ([tokens][H_kv][D], one KV head x
+// 128 keys x 64 columns per box); the paged cache stands in when there is
+// no prefix at all (the maps are then never used).
+inline cudaError_t make_prefix_maps(const AttnParams &p, CUtensorMap *tk, CUtensorMap *tv) {
+  const int D = p.D;
   const bool has_prefix = p.prefix_tokens > 0;
   const uint64_t T = has_prefix ? static_cast<uint64_t>(p.prefix_tokens) : 1;
-  e = make_map(tk, has_prefix ? p.prefix_k : p.k_cache, D, p.H_kv, T, 64, 1, kBlk);
+  cudaError_t e = make_map(tk, has_prefix ? p.prefix_k : p.k_cache, D, p.H_kv, T, 64, 1, kBlk);
   if (e != cudaSuccess) return e;
   return make_map(tv, has_prefix ? p.prefix_v : p.v_cache, D, p.H_kv, T, 64, 1, kBlk);
 }
