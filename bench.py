@@ -172,6 +172,29 @@ def dist_env():
     return world, rank, local
 
 
+def rank_seeds(cid: int, rank: int):
+    """Seeds of a rank's workload (tensors, logits).  Every rank runs its own
+    independent pages (pages never share keys), so ranks draw distinct data."""
+    return 1000 + cid + 100 * rank, 2000 + cid + 100 * rank
+
+
+def max_over_ranks(ms: float, world: int, device) -> float:
+    """The slowest rank's time: all-reduce MAX over the process group."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_value(world: int, qtok_per_rank: int, ms_per_step: float) -> float:
+    """Query tokens all ranks processed per second (weak scaling: each rank
+    processes qtok_per_rank per step, ms_per_step is the max over ranks)."""
+    return world * qtok_per_rank / (ms_per_step * 1e-3)
+
+
 # ------------------------------------------------------------- CPU oracle --
 
 def oracle_sample_run(inp, logits, drafts, budget_s: float, rng_seed: int = 0):
@@ -222,8 +245,9 @@ def run_ours(args, world, rank, local):
     H.load()
 
     cid = int(args.workload.lstrip("c"))
-    inp = W.make_config(args.workload, seed=1000 + cid + 100 * rank)
-    logits_np = W.make_logits(inp.B, inp.m, VOCAB, seed=2000 + cid + 100 * rank)
+    seed_t, seed_l = rank_seeds(cid, rank)
+    inp = W.make_config(args.workload, seed=seed_t)
+    logits_np = W.make_logits(inp.B, inp.m, VOCAB, seed=seed_l)
     stream = torch.cuda.Stream(device=dev)
     sh = int(stream.cuda_stream)
 
@@ -320,10 +344,8 @@ def run_ours(args, world, rank, local):
         wall_ms[0] = (time.perf_counter() - w0) * 1e3
         ms = t0.elapsed_time(t1)
         if world > 1 and sync_ranks:
-            t = torch.tensor([ms], dtype=torch.float64, device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms = max_over_ranks(ms, world, dev)
             dist.barrier()
-            ms = float(t.item())
         return ms
 
     gpu_id = str(torch.cuda.get_device_properties(dev).uuid)
@@ -413,8 +435,8 @@ def run_ours(args, world, rank, local):
 
     qtok = inp.B * inp.m
     ms_step = total_ms / K
-    value = world * qtok / (ms_step * 1e-3)
-    e2e_value = world * qtok / (e2e_ms / K * 1e-3)
+    value = whole_job_value(world, qtok, ms_step)
+    e2e_value = whole_job_value(world, qtok, e2e_ms / K)
 
     pk = peaks()
     per, step_work = algorithmic_work(inp)
