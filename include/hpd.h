@@ -197,6 +197,17 @@ hpd_status hpd_branch_attn_noalloc(const hpd_branch_attn_args *args, hpd_stream_
  * one call that synchronises: it waits for `stream`. */
 hpd_status hpd_read_errors(const void *workspace, uint32_t *flags, hpd_stream_t stream);
 
+/* Self-test of the bounded device waits (no counterpart in the paper): one
+ * warp waits on an mbarrier phase that nothing completes and on a
+ * shared-memory flag that nothing sets, each for about limit_us
+ * microseconds (1 .. 10,000,000), then returns normally.  Each wait that gave
+ * up sets a bit in the workspace error word: HPD_DEVERR_TIMEOUT for the
+ * mbarrier and HPD_DEVERR_TIMEOUT << 8 for the flag.  workspace: device
+ * pointer, 256-byte aligned, at least 256 bytes; the caller clears it first
+ * (hpd_workspace_init) and reads it with hpd_read_errors.  Asynchronous on
+ * `stream`; HPD_ERR_INVALID_ARG for a bad pointer or limit. */
+hpd_status hpd_wait_selftest(void *workspace, uint32_t limit_us, hpd_stream_t stream);
+
 /* Static description of a status code. */
 const char *hpd_status_string(hpd_status status);
 

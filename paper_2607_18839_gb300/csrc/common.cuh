@@ -121,6 +121,7 @@ namespace hpd {
 cudaError_t launch_prefix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
 cudaError_t launch_branch_attn_tc(const AttnParams &p, const Plan &plan, cudaStream_t s);
 cudaError_t launch_merge_splits(const AttnParams &p, cudaStream_t s);
+cudaError_t launch_wait_selftest(uint32_t *err, uint64_t limit_ns, cudaStream_t s);
 cudaError_t launch_suffix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
 // Remember `e` for hpd_last_cuda_error() and return HPD_ERR_CUDA.
 hpd_status record_cuda_error(cudaError_t e);

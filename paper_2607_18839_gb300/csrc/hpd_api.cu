@@ -253,6 +253,15 @@ hpd_status hpd_read_errors(const void *workspace, uint32_t *flags, hpd_stream_t 
   return e == cudaSuccess ? HPD_OK : cuda_fail(e);
 }
 
+hpd_status hpd_wait_selftest(void *workspace, uint32_t limit_us, hpd_stream_t stream) {
+  if (!workspace || !aligned(workspace, kAlign) || limit_us < 1 || limit_us > 10000000u)
+    return HPD_ERR_INVALID_ARG;
+  const cudaError_t e = hpd::launch_wait_selftest(static_cast<uint32_t *>(workspace),
+                                                  static_cast<uint64_t>(limit_us) * 1000u,
+                                                  reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? HPD_OK : cuda_fail(e);
+}
+
 const char *hpd_status_string(hpd_status status) {
   switch (status) {
     case HPD_OK: return "ok";

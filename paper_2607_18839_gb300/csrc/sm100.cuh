@@ -62,19 +62,22 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parit
 // Slow path of mbar_wait: sleep-wait until the phase completes (true), the
 // time limit passes or *abort becomes non-zero (false).  Kept out of line so
 // that the clock read cannot be hoisted into the fast path.
-__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, const int *abort) {
+static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, const int *abort,
+                                            uint64_t limit_ns) {
   const uint64_t t0 = globaltimer();
+  const uint32_t nap = limit_ns < 1000000u ? 1000u : 100000u;  // hint, ns
   for (;;) {
-    if (mbar_try_wait_sleep(bar, parity, 100000u)) return true;
+    if (mbar_try_wait_sleep(bar, parity, nap)) return true;
     if (abort && *reinterpret_cast<const volatile int *>(abort)) return false;
-    if (globaltimer() - t0 > kWaitLimitNs) return false;
+    if (globaltimer() - t0 > limit_ns) return false;
   }
 }
 // Wait for the completion of the phase with parity `parity`; false on
-// timeout (or when *abort, if given, becomes non-zero while waiting).
+// timeout (limit_ns) or when *abort, if given, becomes non-zero while waiting.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
-                                          const int *abort = nullptr) {
-  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, abort);
+                                          const int *abort = nullptr,
+                                          uint64_t limit_ns = kWaitLimitNs) {
+  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, abort, limit_ns);
 }
 
 // ----------------------------------------------------------------- TMA --

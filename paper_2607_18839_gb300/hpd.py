@@ -25,7 +25,7 @@ DEVERR = {0x1: "PREFIX_CU", 0x2: "BRANCH_CU", 0x4: "BRANCH_LEN", 0x8: "PAGE_ID",
 # Every entry point declared in include/hpd.h.
 EXPORTS = ("hpd_branch_attn_workspace_size", "hpd_workspace_init", "hpd_branch_attn",
            "hpd_branch_attn_launches", "hpd_branch_attn_kernel_name", "hpd_branch_attn_marked", "hpd_pmtp_accept", "hpd_read_errors", "hpd_status_string", "hpd_last_cuda_error",
-           "hpd_version", "hpd_branch_attn_noalloc")
+           "hpd_version", "hpd_branch_attn_noalloc", "hpd_wait_selftest")
 
 # Scratch bytes built into libhpd for hpd_branch_attn_noalloc.
 NOALLOC_WORKSPACE_BYTES = 32 << 20
@@ -94,6 +94,8 @@ def load(path: str = LIB_PATH):
     lib.hpd_version.argtypes = []
     lib.hpd_branch_attn_noalloc.restype = I
     lib.hpd_branch_attn_noalloc.argtypes = [ctypes.POINTER(hpd_branch_attn_args), P]
+    lib.hpd_wait_selftest.restype = I
+    lib.hpd_wait_selftest.argtypes = [P, ctypes.c_uint32, P]
     _lib = lib
     return lib
 
@@ -159,6 +161,10 @@ def hpd_read_errors(workspace_ptr: int, stream_handle) -> int:
     _check("hpd_read_errors", load().hpd_read_errors(workspace_ptr, ctypes.byref(flags),
                                                       stream_handle))
     return int(flags.value)
+
+
+def hpd_wait_selftest(workspace_ptr: int, limit_us: int, stream_handle) -> None:
+    _check("hpd_wait_selftest", load().hpd_wait_selftest(workspace_ptr, limit_us, stream_handle))
 
 
 def hpd_branch_attn_noalloc(args: hpd_branch_attn_args, stream_handle: Optional[int]) -> None:
