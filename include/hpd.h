@@ -61,6 +61,7 @@ typedef enum {
 #define HPD_DEVERR_PAGE_ID 0x8u     /* a page id outside [0, num_pages) */
 #define HPD_DEVERR_FORK_LEN 0x10u   /* branch_prefix_len < 0 or > P_d */
 #define HPD_DEVERR_TIMEOUT 0x40u    /* a bounded device-side wait expired */
+#define HPD_DEVERR_POOL 0x80u       /* KV append / rollback: free-page stack short or inconsistent */
 
 /* Tokens per KV page of the paged private cache. */
 #define HPD_PAGE_TOKENS 16
@@ -196,6 +197,48 @@ hpd_status hpd_branch_attn_noalloc(const hpd_branch_attn_args *args, hpd_stream_
 /* Copy the workspace error word (HPD_DEVERR_* bits) to *flags.  This is the
  * one call that synchronises: it waits for `stream`. */
 hpd_status hpd_read_errors(const void *workspace, uint32_t *flags, hpd_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Paged private KV around a decode step (Algorithm 1: the step's tokens are
+ * written to the cache before attention -- WriteKV -- and after verification
+ * the branch keeps what was accepted; the printed length update is garbled,
+ * read here as "keep n_acc + 1 of the step's m rows, roll back the rest").
+ *
+ * Free pages live on a device stack: free_pages[0 .. *free_top) hold page ids
+ * not used by any branch.  Logical page i of branch b is allocated exactly
+ * when i < ceil(branch_len[b] / 16).  Allocation is deterministic (branch
+ * order), all or nothing: on a short stack or a branch that would outgrow
+ * max_pages * 16 rows, nothing changes and the workspace error word gets
+ * HPD_DEVERR_POOL / HPD_DEVERR_BRANCH_LEN.  Device pointers; the caller owns
+ * everything; calls are asynchronous on `stream`.
+ * ------------------------------------------------------------------------ */
+typedef struct {
+  const void *k_new;    /* bf16 [B][m][H_kv][D]: the step's new keys (append) */
+  const void *v_new;    /* bf16 [B][m][H_kv][D]: the step's new values (append) */
+  void *k_cache;        /* bf16 [num_pages][16][H_kv][D], 16-byte aligned */
+  void *v_cache;        /* bf16 [num_pages][16][H_kv][D], 16-byte aligned */
+  int32_t *page_table;  /* [B][max_pages]; freed entries become -1 */
+  int32_t *branch_len;  /* [B], updated in place */
+  int32_t *free_pages;  /* [num_pages] stack of free page ids */
+  int32_t *free_top;    /* [1] number of ids on the stack */
+  void *workspace;      /* 256-byte aligned, >= 256 bytes; word 0: HPD_DEVERR_* bits
+                           (cleared by the caller, e.g. hpd_workspace_init), word 1:
+                           1 when the last append allocated */
+  int B, m, H_kv, D;    /* m in 1..64, D in {64, 128} */
+  int num_pages, max_pages;
+} hpd_kv_args;
+
+/* Append: branch b's m rows of k_new / v_new go to private positions
+ * [L_b, L_b + m) (pages opened by them popped from the stack), L_b += m. */
+hpd_status hpd_kv_append(const hpd_kv_args *args, hpd_stream_t stream);
+
+/* Rollback after hpd_pmtp_accept (same stream): of the step's m rows at
+ * [L_b - m, L_b), keep the first min(accepted_len[b] + 1, m) (none when
+ * accepted_len[b] < 0); L_b shrinks accordingly and the pages past the new
+ * length go back onto the stack in branch order.  accepted_len: int32 [B],
+ * device.  k_new / v_new are not used. */
+hpd_status hpd_kv_rollback(const hpd_kv_args *args, const int32_t *accepted_len,
+                           hpd_stream_t stream);
 
 /* Self-test of the bounded device waits (no counterpart in the paper): one
  * warp waits on an mbarrier phase that nothing completes and on a

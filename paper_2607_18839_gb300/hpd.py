@@ -25,7 +25,8 @@ DEVERR = {0x1: "PREFIX_CU", 0x2: "BRANCH_CU", 0x4: "BRANCH_LEN", 0x8: "PAGE_ID",
 # Every entry point declared in include/hpd.h.
 EXPORTS = ("hpd_branch_attn_workspace_size", "hpd_workspace_init", "hpd_branch_attn",
            "hpd_branch_attn_launches", "hpd_branch_attn_kernel_name", "hpd_branch_attn_marked", "hpd_pmtp_accept", "hpd_read_errors", "hpd_status_string", "hpd_last_cuda_error",
-           "hpd_version", "hpd_branch_attn_noalloc", "hpd_wait_selftest")
+           "hpd_version", "hpd_branch_attn_noalloc", "hpd_wait_selftest", "hpd_kv_append",
+           "hpd_kv_rollback")
 
 # Scratch bytes built into libhpd for hpd_branch_attn_noalloc.
 NOALLOC_WORKSPACE_BYTES = 32 << 20
@@ -53,6 +54,20 @@ class hpd_branch_attn_args(ctypes.Structure):
         ("scale", ctypes.c_float),
         ("out", ctypes.c_void_p), ("lse", ctypes.c_void_p),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
+    ]
+
+
+class hpd_kv_args(ctypes.Structure):
+    """Mirror of the C struct of the same name."""
+
+    _fields_ = [
+        ("k_new", ctypes.c_void_p), ("v_new", ctypes.c_void_p),
+        ("k_cache", ctypes.c_void_p), ("v_cache", ctypes.c_void_p),
+        ("page_table", ctypes.c_void_p), ("branch_len", ctypes.c_void_p),
+        ("free_pages", ctypes.c_void_p), ("free_top", ctypes.c_void_p),
+        ("workspace", ctypes.c_void_p),
+        ("B", ctypes.c_int), ("m", ctypes.c_int), ("H_kv", ctypes.c_int), ("D", ctypes.c_int),
+        ("num_pages", ctypes.c_int), ("max_pages", ctypes.c_int),
     ]
 
 
@@ -96,6 +111,10 @@ def load(path: str = LIB_PATH):
     lib.hpd_branch_attn_noalloc.argtypes = [ctypes.POINTER(hpd_branch_attn_args), P]
     lib.hpd_wait_selftest.restype = I
     lib.hpd_wait_selftest.argtypes = [P, ctypes.c_uint32, P]
+    lib.hpd_kv_append.restype = I
+    lib.hpd_kv_append.argtypes = [ctypes.POINTER(hpd_kv_args), P]
+    lib.hpd_kv_rollback.restype = I
+    lib.hpd_kv_rollback.argtypes = [ctypes.POINTER(hpd_kv_args), P, P]
     _lib = lib
     return lib
 
@@ -165,6 +184,15 @@ def hpd_read_errors(workspace_ptr: int, stream_handle) -> int:
 
 def hpd_wait_selftest(workspace_ptr: int, limit_us: int, stream_handle) -> None:
     _check("hpd_wait_selftest", load().hpd_wait_selftest(workspace_ptr, limit_us, stream_handle))
+
+
+def hpd_kv_append(args: hpd_kv_args, stream_handle) -> None:
+    _check("hpd_kv_append", load().hpd_kv_append(ctypes.byref(args), stream_handle))
+
+
+def hpd_kv_rollback(args: hpd_kv_args, accepted_len_ptr: int, stream_handle) -> None:
+    _check("hpd_kv_rollback", load().hpd_kv_rollback(ctypes.byref(args), accepted_len_ptr,
+                                                      stream_handle))
 
 
 def hpd_branch_attn_noalloc(args: hpd_branch_attn_args, stream_handle: Optional[int]) -> None:
@@ -305,3 +333,33 @@ def pmtp_accept(logits, drafts, stream=None):
     hpd_pmtp_accept(_ptr(logits), _ptr(drafts), B, m, V, _ptr(out_tokens), _ptr(acc),
                     _stream_handle(stream))
     return out_tokens, acc
+
+
+class PagedKV:
+    """Device state of the paged private KV (tensors owned here): the caches,
+    the page table, the branch lengths and the free-page stack, plus a
+    256-byte workspace for the error word.  append() / rollback() call the
+    C ABI on it."""
+
+    def __init__(self, k_cache, v_cache, page_table, branch_len, free_pages, free_top, m):
+        import torch
+        self.k_cache, self.v_cache = k_cache, v_cache
+        self.page_table, self.branch_len = page_table, branch_len
+        self.free_pages, self.free_top = free_pages, free_top
+        self.m = m
+        self.workspace = torch.zeros(256, dtype=torch.uint8, device=k_cache.device)
+        B, max_pages = page_table.shape
+        num_pages, _, H_kv, D = k_cache.shape
+        self.args = hpd_kv_args(None, None, _ptr(k_cache), _ptr(v_cache), _ptr(page_table),
+                                _ptr(branch_len), _ptr(free_pages), _ptr(free_top),
+                                _ptr(self.workspace), B, m, H_kv, D, num_pages, max_pages)
+
+    def append(self, k_new, v_new, stream=None):
+        self.args.k_new, self.args.v_new = _ptr(k_new), _ptr(v_new)
+        hpd_kv_append(self.args, _stream_handle(stream))
+
+    def rollback(self, accepted_len, stream=None):
+        hpd_kv_rollback(self.args, _ptr(accepted_len), _stream_handle(stream))
+
+    def errors(self, stream=None) -> int:
+        return hpd_read_errors(_ptr(self.workspace), _stream_handle(stream))

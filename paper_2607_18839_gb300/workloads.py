@@ -237,3 +237,41 @@ def accept_inputs(seed: int = 1005, B: int = 256, m: int = 4, V: int = 32000):
     """Logits for the c5 acceptance step (drafts are mixed in by the caller
     from the row argmax it trusts, via :func:`mix_drafts`)."""
     return make_logits(B, m, V, seed)
+
+
+# ---------------------------------------------------------- paged KV pool --
+
+def make_kv_pool(lengths, m: int, H_kv: int, D: int, num_pages: int, max_pages: int,
+                 seed: int):
+    """A seeded paged-KV pool: random bf16 caches, each branch's first
+    ceil(L_b / 16) logical pages on distinct random physical pages (the rest
+    of its table row -1), and the unused page ids, shuffled, on the free
+    stack ``free[0:top]``.  Returns a dict of numpy arrays and ``top``."""
+    rng = np.random.default_rng(seed)
+    lengths = np.asarray(lengths, dtype=np.int32)
+    B = lengths.shape[0]
+    used = [(int(l) + PAGE - 1) // PAGE for l in lengths]
+    if sum(used) > num_pages:
+        raise ValueError("pool too small for the lengths")
+    perm = rng.permutation(num_pages).astype(np.int32)
+    page_table = np.full((B, max_pages), -1, dtype=np.int32)
+    at = 0
+    for b in range(B):
+        page_table[b, :used[b]] = perm[at:at + used[b]]
+        at += used[b]
+    free = np.zeros(num_pages, dtype=np.int32)
+    rest = perm[at:]
+    free[:rest.shape[0]] = rest
+    shape = (num_pages, PAGE, H_kv, D)
+    return dict(
+        k_cache=f32_to_bf16_bits(rng.standard_normal(shape, dtype=np.float32) * 0.5),
+        v_cache=f32_to_bf16_bits(rng.standard_normal(shape, dtype=np.float32) * 0.5),
+        page_table=page_table, branch_len=lengths.copy(), free=free, top=int(rest.shape[0]))
+
+
+def make_kv_rows(B: int, m: int, H_kv: int, D: int, seed: int):
+    """bf16 bits [B, m, H_kv, D] of a step's new keys and values."""
+    rng = np.random.default_rng(seed)
+    shape = (B, m, H_kv, D)
+    return (f32_to_bf16_bits(rng.standard_normal(shape, dtype=np.float32) * 0.5),
+            f32_to_bf16_bits(rng.standard_normal(shape, dtype=np.float32) * 0.5))
