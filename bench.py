@@ -382,6 +382,38 @@ def run_ours(args, world, rank, local):
     kernel_ms = {name: attn_ms * span[k] / sum(span) for k, name in enumerate(attn_names)}
     kernel_ms[ACCEPT] = acc_ms
 
+    # ---- paged-KV append / rollback around a step (reported beside the step,
+    # not part of its metric): append the step's m rows of every branch, then
+    # roll all of them back (accepted_len = -1), which restores the pool
+    used = np.ceil(inp.branch_len / W.PAGE).astype(np.int64)
+    kv_max_pages = int(np.max(np.ceil((inp.branch_len + inp.m) / W.PAGE)))
+    kv_pages = int(used.sum() + inp.B * (inp.m // W.PAGE + 2))
+    pool = W.make_kv_pool(inp.branch_len, inp.m, inp.H_kv, inp.D, kv_pages, kv_max_pages,
+                          seed=4000 + cid)
+    kv_new = W.make_kv_rows(inp.B, inp.m, inp.H_kv, inp.D, seed=5000 + cid)
+    tdev = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    kv = H.PagedKV(tdev(pool["k_cache"].view(np.int16)), tdev(pool["v_cache"].view(np.int16)),
+                   tdev(pool["page_table"]), tdev(pool["branch_len"]), tdev(pool["free"]),
+                   torch.tensor([pool["top"]], dtype=torch.int32, device=dev), inp.m)
+    k_new, v_new = (tdev(a.view(np.int16)) for a in kv_new)
+    reject_all = torch.full((inp.B,), -1, dtype=torch.int32, device=dev)
+
+    def kv_pair(r, i):
+        kv.append(k_new, v_new, stream)
+        kv.rollback(reject_all, stream)
+
+    with torch.cuda.stream(stream):
+        kv_pair(0, 0)
+    g_kv = capture(S, 0, kv_pair)
+    kv_ms = timed(g_kv, None, n_rep, sync_ranks=False) / (n_rep * S)
+    if kv.errors(stream):
+        raise SystemExit(f"bench.py: KV append / rollback error flags {kv.errors(stream):#x}")
+    kv_bytes = 2 * 2 * inp.B * inp.m * inp.H_kv * inp.D * 2  # K and V rows read + written
+    kv_line = {"us_per_pair": kv_ms * 1e3, "launches_per_pair": 3, "bytes": kv_bytes,
+               "achieved_gbs": kv_bytes / (kv_ms * 1e-3) / 1e9,
+               "note": "hpd_kv_append (m rows per branch) + hpd_kv_rollback (all rolled back) "
+                       "on a pool of the workload's lengths; not part of the step metric"}
+
     # ---- end to end: pinned host inputs in, results out, every step
     host_q = torch.from_numpy(inp.q.view(np.int16)).pin_memory()
     host_meta = [torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).pin_memory()
@@ -484,6 +516,7 @@ def run_ours(args, world, rank, local):
                           "frac": t_roof / (ms_step * 1e-3)},
         "kernel_us": {k: v * 1e3 for k, v in kernel_ms.items()},
         "attn_call_us": attn_ms * 1e3,
+        "kv_append_rollback": kv_line,
         "host_wall_ms_per_step": total_wall_ms / K,
         "cpu_baseline": cpu,
         "clocks": clk,
