@@ -414,6 +414,35 @@ def run_ours(args, world, rank, local):
                "note": "hpd_kv_append (m rows per branch) + hpd_kv_rollback (all rolled back) "
                        "on a pool of the workload's lengths; not part of the step metric"}
 
+    # ---- fork detection / child branches after the acceptance (reported beside
+    # the step): the step's argmax tokens with 2% fork tokens, each page's
+    # first branch its layout branch
+    rng_f = np.random.default_rng(6000 + cid)
+    fork_tok = np.where(rng_f.random((inp.B, inp.m)) < 0.02, VOCAB - 1,
+                        rng_f.integers(0, VOCAB - 1, size=(inp.B, inp.m))).astype(np.int32)
+    is_layout = np.zeros(inp.B, np.int32)
+    is_layout[inp.branch_cu[:-1][np.diff(inp.branch_cu) > 0]] = 1
+    f_in = [tdev(a) for a in (fork_tok, acc.cpu().numpy(), is_layout,
+                               inp.branch_prefix_len if inp.branch_prefix_len is not None
+                               else np.zeros(inp.B, np.int32), inp.branch_cu, inp.branch_len,
+                               inp.page_table)]
+    f_cap = inp.B * (inp.m + 1)
+    f_state = {}
+
+    def fork_call(r, i):
+        f_state["out"] = H.fork_children(f_in[0], f_in[1], f_in[2], f_in[3], VOCAB - 1, f_in[4],
+                                         None, f_in[5], f_in[6], f_cap, stream)
+
+    with torch.cuda.stream(stream):
+        fork_call(0, 0)
+    torch.cuda.synchronize(dev)
+    g_fork = capture(S, 0, fork_call)
+    fork_ms = timed(g_fork, None, n_rep, sync_ranks=False) / (n_rep * S)
+    fork_line = {"us_per_call": fork_ms * 1e3,
+                 "children": int(f_state["out"]["new_B"].item()) - inp.B,
+                 "note": "hpd_fork_children over the step's branches (two launches); not part of "
+                         "the step metric"}
+
     # ---- end to end: pinned host inputs in, results out, every step
     host_q = torch.from_numpy(inp.q.view(np.int16)).pin_memory()
     host_meta = [torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).pin_memory()
@@ -517,6 +546,7 @@ def run_ours(args, world, rank, local):
         "kernel_us": {k: v * 1e3 for k, v in kernel_ms.items()},
         "attn_call_us": attn_ms * 1e3,
         "kv_append_rollback": kv_line,
+        "fork_children": fork_line,
         "host_wall_ms_per_step": total_wall_ms / K,
         "cpu_baseline": cpu,
         "clocks": clk,

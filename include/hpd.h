@@ -62,6 +62,7 @@ typedef enum {
 #define HPD_DEVERR_FORK_LEN 0x10u   /* branch_prefix_len < 0 or > P_d */
 #define HPD_DEVERR_TIMEOUT 0x40u    /* a bounded device-side wait expired */
 #define HPD_DEVERR_POOL 0x80u       /* KV append / rollback: free-page stack short or inconsistent */
+#define HPD_DEVERR_FORK_CAP 0x100u  /* fork: more branches than the output capacity */
 
 /* Tokens per KV page of the paged private cache. */
 #define HPD_PAGE_TOKENS 16
@@ -239,6 +240,53 @@ hpd_status hpd_kv_append(const hpd_kv_args *args, hpd_stream_t stream);
  * device.  k_new / v_new are not used. */
 hpd_status hpd_kv_rollback(const hpd_kv_args *args, const int32_t *accepted_len,
                            hpd_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Fork detection and child branches after verification (Algorithm 1: scan
+ * the accepted tokens for the fork token, spawn a child sharing the parent's
+ * context; Sec. 3.3).  A page's shared context is its prefix (vision tokens,
+ * then its layout branch's tokens), so a child is a new branch of the same
+ * page whose fork-position prefix length is just past the fork token, with
+ * no private keys: nothing is copied.
+ *
+ * A layout branch b (is_layout[b] != 0, or every branch when is_layout is
+ * NULL) emits out_tokens[b][0 .. e_b), e_b = min(accepted_len[b] + 1, m)
+ * (accepted drafts, then the correction token); token i sits at prefix
+ * position layout_pos[b] + i.  Each emitted fork token spawns a child with
+ * prefix length layout_pos[b] + i + 1, private length 0 and an all -1 page
+ * table row.  Outputs (device, capacity `cap` branches): the branch arrays of
+ * the new set, each page's old branches first (in order), then its children
+ * in (parent, index) order; new_parent[i] = the old index of an old branch,
+ * or -1 - parent for a child; new_branch_prefix_len of an old branch is its
+ * branch_prefix_len (-1 when that array is NULL: the whole page prefix).
+ * *new_B = the new branch count, or -1 with HPD_DEVERR_FORK_CAP in the
+ * workspace error word when it would exceed cap (the outputs are then not
+ * written).  workspace: 256-byte aligned, >= 4 * (65 + n_docs) bytes, word 0
+ * the error word (cleared by the caller).  Two launches (a one-CTA scan, then
+ * the copy of the old branches' arrays), asynchronous on `stream`.
+ * ------------------------------------------------------------------------ */
+typedef struct {
+  const int32_t *out_tokens;         /* [B][m] (hpd_pmtp_accept) */
+  const int32_t *accepted_len;       /* [B] */
+  const int32_t *is_layout;          /* [B] or NULL */
+  const int32_t *layout_pos;         /* [B] prefix position of the step's token 0 */
+  const int32_t *branch_cu;          /* [n_docs + 1], monotone, branch_cu[n_docs] = B */
+  const int32_t *branch_prefix_len;  /* [B] or NULL */
+  const int32_t *branch_len;         /* [B] */
+  const int32_t *page_table;         /* [B][max_pages] */
+  int32_t *new_branch_cu;            /* [n_docs + 1] */
+  int32_t *new_branch_prefix_len;    /* [cap] */
+  int32_t *new_branch_len;           /* [cap] */
+  int32_t *new_page_table;           /* [cap][max_pages] */
+  int32_t *new_parent;               /* [cap] */
+  int32_t *new_B;                    /* [1] */
+  void *workspace;
+  size_t workspace_bytes;
+  int32_t fork_token;
+  int B, m, n_docs, max_pages, cap;
+} hpd_fork_args;
+
+hpd_status hpd_fork_children(const hpd_fork_args *args, hpd_stream_t stream);
 
 /* Self-test of the bounded device waits (no counterpart in the paper): one
  * warp waits on an mbarrier phase that nothing completes and on a

@@ -26,7 +26,7 @@ DEVERR = {0x1: "PREFIX_CU", 0x2: "BRANCH_CU", 0x4: "BRANCH_LEN", 0x8: "PAGE_ID",
 EXPORTS = ("hpd_branch_attn_workspace_size", "hpd_workspace_init", "hpd_branch_attn",
            "hpd_branch_attn_launches", "hpd_branch_attn_kernel_name", "hpd_branch_attn_marked", "hpd_pmtp_accept", "hpd_read_errors", "hpd_status_string", "hpd_last_cuda_error",
            "hpd_version", "hpd_branch_attn_noalloc", "hpd_wait_selftest", "hpd_kv_append",
-           "hpd_kv_rollback")
+           "hpd_kv_rollback", "hpd_fork_children")
 
 # Scratch bytes built into libhpd for hpd_branch_attn_noalloc.
 NOALLOC_WORKSPACE_BYTES = 32 << 20
@@ -69,6 +69,18 @@ class hpd_kv_args(ctypes.Structure):
         ("B", ctypes.c_int), ("m", ctypes.c_int), ("H_kv", ctypes.c_int), ("D", ctypes.c_int),
         ("num_pages", ctypes.c_int), ("max_pages", ctypes.c_int),
     ]
+
+
+class hpd_fork_args(ctypes.Structure):
+    """Mirror of the C struct of the same name."""
+
+    _fields_ = [(n, ctypes.c_void_p) for n in (
+        "out_tokens", "accepted_len", "is_layout", "layout_pos", "branch_cu", "branch_prefix_len",
+        "branch_len", "page_table", "new_branch_cu", "new_branch_prefix_len", "new_branch_len",
+        "new_page_table", "new_parent", "new_B", "workspace")] + [
+        ("workspace_bytes", ctypes.c_size_t), ("fork_token", ctypes.c_int32),
+        ("B", ctypes.c_int), ("m", ctypes.c_int), ("n_docs", ctypes.c_int),
+        ("max_pages", ctypes.c_int), ("cap", ctypes.c_int)]
 
 
 _lib = None
@@ -115,6 +127,8 @@ def load(path: str = LIB_PATH):
     lib.hpd_kv_append.argtypes = [ctypes.POINTER(hpd_kv_args), P]
     lib.hpd_kv_rollback.restype = I
     lib.hpd_kv_rollback.argtypes = [ctypes.POINTER(hpd_kv_args), P, P]
+    lib.hpd_fork_children.restype = I
+    lib.hpd_fork_children.argtypes = [ctypes.POINTER(hpd_fork_args), P]
     _lib = lib
     return lib
 
@@ -363,3 +377,32 @@ class PagedKV:
 
     def errors(self, stream=None) -> int:
         return hpd_read_errors(_ptr(self.workspace), _stream_handle(stream))
+
+
+def fork_children(out_tokens, accepted_len, is_layout, layout_pos, fork_token, branch_cu,
+                  branch_prefix_len, branch_len, page_table, cap, stream=None):
+    """Device tensors in (int32); returns a dict of new device tensors
+    (branch_cu, branch_prefix_len, branch_len, page_table, parent, new_B,
+    workspace) with capacity `cap` branches."""
+    import torch
+    dev = out_tokens.device
+    B, m = out_tokens.shape
+    n_docs = branch_cu.shape[0] - 1
+    max_pages = page_table.shape[1]
+    new = dict(branch_cu=torch.empty(n_docs + 1, dtype=torch.int32, device=dev),
+               branch_prefix_len=torch.empty(cap, dtype=torch.int32, device=dev),
+               branch_len=torch.empty(cap, dtype=torch.int32, device=dev),
+               page_table=torch.empty((cap, max_pages), dtype=torch.int32, device=dev),
+               parent=torch.empty(cap, dtype=torch.int32, device=dev),
+               new_B=torch.empty(1, dtype=torch.int32, device=dev))
+    ws_bytes = max(256, 4 * (65 + n_docs))
+    ws_bytes = (ws_bytes + 255) // 256 * 256
+    new["workspace"] = torch.zeros(ws_bytes, dtype=torch.uint8, device=dev)
+    args = hpd_fork_args(_ptr(out_tokens), _ptr(accepted_len), _ptr(is_layout), _ptr(layout_pos),
+                         _ptr(branch_cu), _ptr(branch_prefix_len), _ptr(branch_len),
+                         _ptr(page_table), _ptr(new["branch_cu"]), _ptr(new["branch_prefix_len"]),
+                         _ptr(new["branch_len"]), _ptr(new["page_table"]), _ptr(new["parent"]),
+                         _ptr(new["new_B"]), _ptr(new["workspace"]), ws_bytes, fork_token, B, m,
+                         n_docs, max_pages, cap)
+    _check("hpd_fork_children", load().hpd_fork_children(ctypes.byref(args), _stream_handle(stream)))
+    return new

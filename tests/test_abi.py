@@ -86,3 +86,32 @@ def test_accept_rejects_bad_arguments_before_launch(lib):
     with pytest.raises(hpd.HpdError) as e:
         hpd.hpd_pmtp_accept(16, 16, 4, 65, 100, 16, 16, None)
     assert e.value.status == 2
+
+
+def test_struct_layouts_match_the_header(tmp_path):
+    """sizeof / offsetof of the C structs, compiled from include/hpd.h, equal
+    the ctypes mirrors of the binding."""
+    import shutil
+    import subprocess
+    if shutil.which("gcc") is None:
+        pytest.skip("no gcc")
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    src = tmp_path / "layout.c"
+    src.write_text(
+        '#include <stdio.h>\n#include <stddef.h>\n#include "hpd.h"\n'
+        'int main(void) {\n'
+        '  printf("%zu %zu %zu\\n", sizeof(hpd_branch_attn_args), offsetof(hpd_branch_attn_args, out),'
+        ' offsetof(hpd_branch_attn_args, workspace_bytes));\n'
+        '  printf("%zu %zu %zu\\n", sizeof(hpd_kv_args), offsetof(hpd_kv_args, workspace),'
+        ' offsetof(hpd_kv_args, max_pages));\n'
+        '  printf("%zu %zu %zu\\n", sizeof(hpd_fork_args), offsetof(hpd_fork_args, fork_token),'
+        ' offsetof(hpd_fork_args, cap));\n'
+        '  return 0;\n}\n')
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-I", os.path.join(root, "include"), str(src), "-o", str(exe)], check=True)
+    got = [list(map(int, l.split())) for l in subprocess.run([str(exe)], capture_output=True,
+                                                              text=True, check=True).stdout.split("\n") if l]
+    A, K, F = hpd.hpd_branch_attn_args, hpd.hpd_kv_args, hpd.hpd_fork_args
+    assert got[0] == [ctypes.sizeof(A), A.out.offset, A.workspace_bytes.offset]
+    assert got[1] == [ctypes.sizeof(K), K.workspace.offset, K.max_pages.offset]
+    assert got[2] == [ctypes.sizeof(F), F.fork_token.offset, F.cap.offset]
