@@ -142,8 +142,9 @@ const char *hpd_branch_attn_kernel_name(const hpd_branch_attn_args *args, int k)
 /* hpd_branch_attn with timing markers.  stage_events holds
  * hpd_branch_attn_launches(args) + 1 cudaEvent_t handles created by the
  * caller (with timing enabled); event 0 is recorded on `stream` before the
- * first kernel and event k after the k-th.  Recorded as external events, so
- * they also work inside stream capture.  NULL behaves as hpd_branch_attn. */
+ * first kernel and event k after the k-th.  While `stream` is capturing they
+ * are recorded as external event nodes (so a replayed graph times each
+ * kernel), otherwise as plain records.  NULL behaves as hpd_branch_attn. */
 hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *args, hpd_stream_t stream,
                                   void *const *stage_events);
 

@@ -244,6 +244,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) u = atomicAdd(p.unit_ctr, 1);
         u = __shfl_sync(0xffffffffu, u, 0);
         if (u >= p.n_units || aborted(sh)) break;
+        if (p.unit_order) u = p.unit_order[u];  // longest units first
         const int split = u % p.S_p;
         const int g = (u / p.S_p) % p.H_kv;
         const int tile = u / (p.S_p * p.H_kv);

@@ -25,10 +25,12 @@ struct Plan {
   int wr_s;        // warps along rows in the suffix kernel (1, 2, 4)
   int rt_s;        // suffix row tiles per (branch, KV head)
   bool use_tc;     // whole step on tcgen05 (G divides 128) or warp MMA stages
+  bool lpt;        // tcgen05: order the units longest first (more units than SMs)
   size_t off_err;    // uint32 error word
   size_t off_ctr;    // int32 tickets [B][H_kv][rt_s]
   size_t off_opart;  // fp32 [S_p + S_s][rows_total][H_q][D]
   size_t off_lpart;  // fp32 [S_p + S_s][rows_total][H_q]
+  size_t off_order;  // int32 [n_units] unit order (lpt)
   size_t bytes;      // total workspace bytes
 };
 
@@ -54,6 +56,7 @@ struct AttnParams {
   int *counters;        // per (branch, KV head, row tile) arrival tickets, zero between calls
   int *unit_ctr;        // [2] persistent-kernel unit counter and finished-CTA count, zero between calls
   int n_units;          // work units of the tcgen05 kernel (row tile x KV head x split)
+  const int *unit_order;  // the order in which to take them (null: index order)
   __nv_bfloat16 *out;   // final output, written by the suffix stage
   float *lse;           // final lse (may be null)
 };
@@ -120,6 +123,8 @@ __device__ __forceinline__ int ceil_div_i(int a, int b) { return (a + b - 1) / b
 namespace hpd {
 cudaError_t launch_prefix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
 cudaError_t launch_branch_attn_tc(const AttnParams &p, const Plan &plan, cudaStream_t s);
+cudaError_t launch_unit_order(const AttnParams &p, int tiles, int *order, cudaStream_t s);
+size_t unit_order_smem_bytes(int n_docs, int B, int tiles);
 cudaError_t launch_merge_splits(const AttnParams &p, cudaStream_t s);
 cudaError_t launch_wait_selftest(uint32_t *err, uint64_t limit_ns, cudaStream_t s);
 cudaError_t launch_suffix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);

@@ -22,6 +22,8 @@ constexpr int kPlanSms = 152;          // SMs the split plan assumes (GB300)
 constexpr int kTargetCtas = kPlanSms * 4;  // warp-MMA prefix CTAs aimed for
 constexpr int kTcTileRows = 128;       // stacked rows of one tcgen05 prefix CTA
 constexpr int kMaxPrefixSplits = 8;
+constexpr int kLptWaves = 2;
+constexpr size_t kOrderSmemMax = 200 * 1024;
 constexpr int kSuffixSplitKeys = 1536;  // a suffix chunk holds at most ~this many keys
 constexpr int kMaxSuffixSplits = 8;
 
@@ -86,6 +88,11 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
       }
     }
     pl.S_p = best;
+    // With at least kLptWaves units per SM, units of unequal length leave
+    // SMs idle at the end; a one-CTA pass then orders them longest first
+    // (it holds the per-page and per-branch lengths in shared memory).
+    pl.lpt = ctas * best >= kLptWaves * kPlanSms &&
+             hpd::unit_order_smem_bytes(a->n_docs, a->B, pl.tiles_max) <= kOrderSmemMax;
   } else {
     const long long stacked = static_cast<long long>(a->B) * a->m * pl.G;
     const int tiles = ceil_div(stacked, kPrefixTileRows);
@@ -106,7 +113,10 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
   pl.off_ctr = kAlign;
   pl.off_opart = align_up(pl.off_ctr + static_cast<size_t>(a->B) * a->H_kv * pl.rt_s * sizeof(int));
   pl.off_lpart = align_up(pl.off_opart + S * pairs * a->D * sizeof(float));
-  pl.bytes = align_up(pl.off_lpart + S * pairs * sizeof(float));
+  pl.off_order = align_up(pl.off_lpart + S * pairs * sizeof(float));
+  const size_t n_units =
+      pl.use_tc ? static_cast<size_t>(std::max(pl.tiles_max, 0)) * a->H_kv * pl.S_p : 0;
+  pl.bytes = align_up(pl.off_order + n_units * sizeof(int));
   return pl;
 }
 
@@ -137,17 +147,20 @@ hpd_status hpd_workspace_init(void *workspace, size_t workspace_bytes, hpd_strea
 int hpd_branch_attn_launches(const hpd_branch_attn_args *args) {
   if (check_scalars(args) != HPD_OK) return 0;
   const hpd::Plan pl = make_plan(args);
-  return pl.use_tc ? (pl.S_p > 1 ? 2 : 1) : 2;
+  return pl.use_tc ? 1 + (pl.lpt ? 1 : 0) + (pl.S_p > 1 ? 1 : 0) : 2;
 }
 
 const char *hpd_branch_attn_kernel_name(const hpd_branch_attn_args *args, int k) {
   if (check_scalars(args) != HPD_OK) return nullptr;
   const hpd::Plan pl = make_plan(args);
-  static const char *tc_names[] = {"branch_attn_tc", "merge_splits"};
   static const char *mma_names[] = {"prefix_stage", "suffix_merge"};
-  const int n = pl.use_tc ? (pl.S_p > 1 ? 2 : 1) : 2;
-  if (k < 0 || k >= n) return nullptr;
-  return pl.use_tc ? tc_names[k] : mma_names[k];
+  if (!pl.use_tc) return k >= 0 && k < 2 ? mma_names[k] : nullptr;
+  const char *tc_names[3];
+  int n = 0;
+  if (pl.lpt) tc_names[n++] = "unit_order";
+  tc_names[n++] = "branch_attn_tc";
+  if (pl.S_p > 1) tc_names[n++] = "merge_splits";
+  return k >= 0 && k < n ? tc_names[k] : nullptr;
 }
 
 hpd_status hpd_branch_attn(const hpd_branch_attn_args *a, hpd_stream_t stream) {
@@ -205,21 +218,38 @@ hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t st
   p.counters = reinterpret_cast<int *>(ws + pl.off_ctr);
   p.unit_ctr = reinterpret_cast<int *>(ws + pl.off_err + 8);  // header: err word, then counters
   p.n_units = pl.tiles_max * a->H_kv * pl.S_p;
+  p.unit_order = pl.lpt ? reinterpret_cast<int *>(ws + pl.off_order) : nullptr;
   p.out = static_cast<__nv_bfloat16 *>(a->out);
   p.lse = a->lse;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // inside stream capture an event record becomes an external event node;
+  // outside it, a plain record
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (ev) {
+    const cudaError_t ce = cudaStreamIsCapturing(s, &cap);
+    if (ce != cudaSuccess) return hpd::record_cuda_error(ce);
+  }
   auto mark = [&](int k) -> cudaError_t {
     if (!ev || !ev[k]) return cudaSuccess;
-    return cudaEventRecordWithFlags(static_cast<cudaEvent_t>(ev[k]), s, cudaEventRecordExternal);
+    cudaEvent_t evk = static_cast<cudaEvent_t>(ev[k]);
+    return cap == cudaStreamCaptureStatusActive
+               ? cudaEventRecordWithFlags(evk, s, cudaEventRecordExternal)
+               : cudaEventRecord(evk, s);
   };
   cudaError_t e = mark(0);
   if (pl.use_tc) {
+    int k = 1;
+    if (pl.lpt) {
+      if (e == cudaSuccess)
+        e = hpd::launch_unit_order(p, pl.tiles_max, const_cast<int *>(p.unit_order), s);
+      if (e == cudaSuccess) e = mark(k++);
+    }
     if (e == cudaSuccess) e = hpd::launch_branch_attn_tc(p, pl, s);
-    if (e == cudaSuccess) e = mark(1);
+    if (e == cudaSuccess) e = mark(k++);
     if (pl.S_p > 1) {
       if (e == cudaSuccess) e = hpd::launch_merge_splits(p, s);
-      if (e == cudaSuccess) e = mark(2);
+      if (e == cudaSuccess) e = mark(k++);
     }
   } else {
     if (e == cudaSuccess) e = hpd::launch_prefix_stage(p, pl, s);

@@ -136,6 +136,40 @@ def test_repeated_calls_are_deterministic(hpd):
     assert torch.equal(o1, o2)
 
 
+@pytest.mark.parametrize("name", ["c2", "c4"])
+def test_marked_call_outside_and_inside_capture(hpd, name):
+    """hpd_branch_attn_marked: same results as the plain call, one timed
+    interval per kernel, eager and inside a captured graph."""
+    inp = W.make_config(name)
+    d = hpd.DeviceInputs.from_host(inp)
+    op = hpd.BranchAttn(d)
+    ref = op()[0].clone()
+    n = hpd.hpd_branch_attn_launches(op.args)
+    names = [hpd.hpd_branch_attn_kernel_name(op.args, k) for k in range(n)]
+    assert "branch_attn_tc" in names and hpd.hpd_branch_attn_kernel_name(op.args, n) is None
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
+    for e in ev:
+        e.record()
+    torch.cuda.synchronize()
+    op.out.zero_()
+    op(events=ev)
+    torch.cuda.synchronize()
+    assert torch.equal(op.out, ref)
+    assert all(ev[k].elapsed_time(ev[k + 1]) > 0 for k in range(n))
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        op()  # warm on the capture stream
+        s.synchronize()
+        with torch.cuda.graph(g, stream=s):
+            op(stream=s, events=ev)
+    op.out.zero_()
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(op.out, ref)
+    assert ev[0].elapsed_time(ev[n]) > 0
+
+
 def test_out_of_range_device_data_is_clamped_and_flagged(hpd):
     inp = W.build_inputs([40], [2], [20, 30], 2, 8, 2, 64, seed=39)
     inp.page_table[1, 0] = inp.num_pages + 5   # page id out of range
