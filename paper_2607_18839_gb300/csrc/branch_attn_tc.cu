@@ -226,6 +226,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sh.tmem_base;
+  pdl_wait();     // the unit order (and everything before it) is complete
+  pdl_trigger();  // the merge of the splits may launch; it waits for this grid
 
   if (warp == kSchedWarp) {
     // ------------------------------------------------------- scheduler --
@@ -782,7 +784,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 template <int D>
-cudaError_t launch_tc(const AttnParams &p, cudaStream_t s) {
+cudaError_t launch_tc(const AttnParams &p, bool overlap, cudaStream_t s) {
   using L = TcLayout<D>;
   static_assert(L::kDynSmem + sizeof(TcShared) <= 227 * 1024, "shared memory");
   CUtensorMap tk, tv, tkc, tvc;
@@ -809,15 +811,16 @@ cudaError_t launch_tc(const AttnParams &p, cudaStream_t s) {
     sms[dev & 63] = n;
   }
   const dim3 grid(static_cast<unsigned>(std::min(p.n_units, sms[dev & 63])), 1, 1);
-  branch_attn_tc_kernel<D><<<grid, kThreads, L::kDynSmem, s>>>(tk, tv, tkc, tvc, p);
-  return cudaGetLastError();
+  return launch_kernel(overlap, branch_attn_tc_kernel<D>, grid, dim3(kThreads), L::kDynSmem, s,
+                       tk, tv, tkc, tvc, p);
 }
 
 }  // namespace
 
-cudaError_t launch_branch_attn_tc(const AttnParams &p, const Plan &plan, cudaStream_t s) {
+cudaError_t launch_branch_attn_tc(const AttnParams &p, const Plan &plan, bool overlap,
+                                  cudaStream_t s) {
   if (plan.tiles_max <= 0 || p.n_units <= 0) return cudaSuccess;
-  return p.D == 64 ? launch_tc<64>(p, s) : launch_tc<128>(p, s);
+  return p.D == 64 ? launch_tc<64>(p, overlap, s) : launch_tc<128>(p, overlap, s);
 }
 
 }  // namespace hpd

@@ -117,15 +117,46 @@ __device__ __forceinline__ float fast_exp2(float x) {
 
 __device__ __forceinline__ int ceil_div_i(int a, int b) { return (a + b - 1) / b; }
 
+// Programmatic dependent launch.  A kernel launched with programmatic stream
+// serialization may start while the kernel before it on the stream still
+// runs; pdl_wait() returns once that kernel has finished and its writes are
+// visible (at once when there is no such kernel), so everything the kernel
+// reads from its predecessor comes after it.  pdl_trigger() lets the next
+// such kernel start launching.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Launch `kernel`; with `overlap`, programmatically serialized after the
+// previous kernel on `s` (the kernel must call pdl_wait() before using that
+// kernel's results).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(bool overlap, void (*kernel)(KArgs...), dim3 grid, dim3 block,
+                          size_t smem, cudaStream_t s, Args &&...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = overlap ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
 }  // namespace hpd
 
 // Host-side launchers (defined in the .cu files, called by hpd_api.cu).
 namespace hpd {
 cudaError_t launch_prefix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
-cudaError_t launch_branch_attn_tc(const AttnParams &p, const Plan &plan, cudaStream_t s);
+cudaError_t launch_branch_attn_tc(const AttnParams &p, const Plan &plan, bool overlap,
+                                  cudaStream_t s);
 cudaError_t launch_unit_order(const AttnParams &p, int tiles, int *order, cudaStream_t s);
 size_t unit_order_smem_bytes(int n_docs, int B, int tiles);
-cudaError_t launch_merge_splits(const AttnParams &p, cudaStream_t s);
+cudaError_t launch_merge_splits(const AttnParams &p, bool overlap, cudaStream_t s);
 cudaError_t launch_wait_selftest(uint32_t *err, uint64_t limit_ns, cudaStream_t s);
 cudaError_t launch_suffix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
 // Remember `e` for hpd_last_cuda_error() and return HPD_ERR_CUDA.

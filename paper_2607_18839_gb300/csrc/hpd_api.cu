@@ -245,10 +245,11 @@ hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t st
         e = hpd::launch_unit_order(p, pl.tiles_max, const_cast<int *>(p.unit_order), s);
       if (e == cudaSuccess) e = mark(k++);
     }
-    if (e == cudaSuccess) e = hpd::launch_branch_attn_tc(p, pl, s);
+    // each kernel after the first overlaps its launch with its predecessor
+    if (e == cudaSuccess) e = hpd::launch_branch_attn_tc(p, pl, pl.lpt, s);
     if (e == cudaSuccess) e = mark(k++);
     if (pl.S_p > 1) {
-      if (e == cudaSuccess) e = hpd::launch_merge_splits(p, s);
+      if (e == cudaSuccess) e = hpd::launch_merge_splits(p, true, s);
       if (e == cudaSuccess) e = mark(k++);
     }
   } else {

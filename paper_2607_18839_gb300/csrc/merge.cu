@@ -25,6 +25,7 @@ __global__ void __launch_bounds__(256) merge_splits_kernel(const AttnParams p) {
   const int lane = threadIdx.x & 31;
   const long long n_pairs = static_cast<long long>(p.rows_total) * p.H_q;
   const long long pair = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  pdl_wait();  // the partial results of the attention kernel
   if (pair >= n_pairs) return;
   const float NEG_INF = -__int_as_float(0x7f800000);
   const int S = p.S_p;
@@ -79,16 +80,14 @@ __global__ void __launch_bounds__(256) merge_splits_kernel(const AttnParams p) {
 
 }  // namespace
 
-cudaError_t launch_merge_splits(const AttnParams &p, cudaStream_t s) {
+cudaError_t launch_merge_splits(const AttnParams &p, bool overlap, cudaStream_t s) {
   if (p.S_p > kMaxSplits) return cudaErrorInvalidValue;
   const long long n_pairs = static_cast<long long>(p.rows_total) * p.H_q;
   const long long blocks = (n_pairs * 32 + 255) / 256;
   if (blocks <= 0) return cudaSuccess;
-  if (p.D == 64)
-    merge_splits_kernel<64><<<static_cast<unsigned>(blocks), 256, 0, s>>>(p);
-  else
-    merge_splits_kernel<128><<<static_cast<unsigned>(blocks), 256, 0, s>>>(p);
-  return cudaGetLastError();
+  const dim3 grid(static_cast<unsigned>(blocks));
+  return p.D == 64 ? launch_kernel(overlap, merge_splits_kernel<64>, grid, dim3(256), 0, s, p)
+                   : launch_kernel(overlap, merge_splits_kernel<128>, grid, dim3(256), 0, s, p);
 }
 
 }  // namespace hpd

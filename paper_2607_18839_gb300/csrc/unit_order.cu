@@ -55,6 +55,7 @@ __global__ void __launch_bounds__(kOrderThreads) unit_order_kernel(AttnParams p,
                                                                    int *order) {
   extern __shared__ int sm[];
   __shared__ int ws[33];
+  pdl_trigger();  // the attention kernel may set up meanwhile; it waits for the order
   const int nd = p.n_docs, tid = threadIdx.x;
   int *cnt = sm;                    // [kBuckets]
   int *tile_base = cnt + kBuckets;  // [nd + 1] tiles before page d
