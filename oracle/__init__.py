@@ -13,7 +13,9 @@ Functions
 branch_attn(inp, branch_sel=None, n_threads=0) -> (out fp64, lse fp64)
     Masked-softmax attention of every branch over its shared prefix plus its
     own causal private suffix (Sec. 3.3, "Dynamic Branch Forking and Efficient
-    Context Isolation"; Sec. 3.4 for the m P-MTP queries).
+    Context Isolation"; Sec. 3.4 for the m P-MTP queries).  The prefix is
+    contiguous, or paged in the private keys' pool when the workload carries
+    a ``prefix_page_table``.
 pmtp_accept(logits_bf16, drafts) -> (out_tokens int32, accepted_len int32)
     Greedy verification of the P-MTP drafts (Sec. 3.4; Algorithm 1's
     verification step), lowest index on argmax ties.
@@ -51,7 +53,8 @@ def _load():
         P = ctypes.c_void_p
         I = ctypes.c_int
         lib.oracle_branch_attn.restype = I
-        lib.oracle_branch_attn.argtypes = [P] * 10 + [I] * 8 + [ctypes.c_double, P, I, I, P, P]
+        lib.oracle_branch_attn.argtypes = [P] * 10 + [I] * 8 + [ctypes.c_double, P, I, I, P, P,
+                                                                 P, I]
         lib.oracle_pmtp_accept.restype = None
         lib.oracle_pmtp_accept.argtypes = [P, P, I, I, I, P, P]
         lib.oracle_max_threads.restype = I
@@ -91,6 +94,7 @@ def branch_attn(inp, branch_sel=None, n_threads: int = 0):
         kc=_c(inp.k_cache, np.uint16), vc=_c(inp.v_cache, np.uint16),
         pt=_c(inp.page_table, np.int32), bl=_c(inp.branch_len, np.int32),
         sel=_c(branch_sel, np.int32),
+        ppt=_c(getattr(inp, "prefix_page_table", None), np.int32),
     )
     scale = inp.scale if inp.scale else 1.0 / np.sqrt(inp.D)
     n_sel = 0 if branch_sel is None else len(arrs["sel"])
@@ -98,7 +102,8 @@ def branch_attn(inp, branch_sel=None, n_threads: int = 0):
         _ptr(arrs["q"]), _ptr(arrs["pk"]), _ptr(arrs["pv"]), _ptr(arrs["pcu"]), _ptr(arrs["bcu"]),
         _ptr(arrs["bpl"]), _ptr(arrs["kc"]), _ptr(arrs["vc"]), _ptr(arrs["pt"]), _ptr(arrs["bl"]),
         inp.n_docs, inp.B, inp.m, inp.H_q, inp.H_kv, inp.D, inp.num_pages, inp.max_pages,
-        float(scale), _ptr(arrs["sel"]), n_sel, int(n_threads), _ptr(out), _ptr(lse))
+        float(scale), _ptr(arrs["sel"]), n_sel, int(n_threads), _ptr(out), _ptr(lse),
+        _ptr(arrs["ppt"]), 0 if arrs["ppt"] is None else int(arrs["ppt"].shape[1]))
     if rc != 0:
         raise ValueError("oracle_branch_attn: an index falls outside its buffer")
     return out, lse

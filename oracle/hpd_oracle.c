@@ -23,6 +23,12 @@
  *        private keys  j in [0, L_b - m + i]         (L_b includes the m
  *                                                     tokens of this step)
  *     Private key j lives in physical page page_table[b][j / 16], slot j % 16.
+ *     The prefix is either contiguous (page d's keys are rows
+ *     [prefix_cu[d], prefix_cu[d+1]) of prefix_k / prefix_v) or paged in the
+ *     same pool as the private keys, shared by every branch of the page
+ *     without a copy (Algorithm 1's fork shares the parent's KV pages):
+ *     prefix key j of page d is slot j % 16 of physical page
+ *     prefix_page_table[d][j / 16].
  *     With s_j = scale * <q, k_j> over the visible set K:
  *        M   = max_j s_j
  *        out = sum_j exp(s_j - M) v_j / sum_j exp(s_j - M)
@@ -76,6 +82,9 @@ int oracle_max_threads(void) {
  * page_table [B][max_pages]
  * branch_len [B]                     L_b, private entries incl. this step's m
  * branch_sel [n_sel] or NULL         compute only these branches (NULL: all)
+ * prefix_page_table [n_docs][max_prefix_pages] or NULL
+ *                                    paged prefix in k_cache / v_cache;
+ *                                    prefix_k / prefix_v are then unused
  * out [B*m][H_q][D], lse [B*m][H_q]  written only for the computed branches
  *
  * Returns 0, or -1 on an index that falls outside its buffer.
@@ -89,7 +98,8 @@ int oracle_branch_attn(const uint16_t *q, const uint16_t *prefix_k,
                        int n_docs, int B, int m, int H_q, int H_kv, int D,
                        int num_pages, int max_pages, double scale,
                        const int32_t *branch_sel, int n_sel, int n_threads,
-                       double *out, double *lse) {
+                       double *out, double *lse, const int32_t *prefix_page_table,
+                       int max_prefix_pages) {
   if (H_kv <= 0 || H_q % H_kv != 0) return -1;
   const int G = H_q / H_kv;
   const int n_branches = branch_sel ? n_sel : B;
@@ -115,6 +125,22 @@ int oracle_branch_attn(const uint16_t *q, const uint16_t *prefix_k,
     const int P_d = prefix_cu[d + 1] - prefix_cu[d];
     int P_b = branch_prefix_len ? branch_prefix_len[b] : P_d;
     if (P_b < 0 || P_b > P_d) { bad = 1; continue; }
+    if (prefix_page_table && P_d > max_prefix_pages * ORACLE_PAGE) { bad = 1; continue; }
+    /* K and V of prefix key j: a row of prefix_k / prefix_v, or a page slot */
+    const uint16_t *pk_base = prefix_page_table ? k_cache : prefix_k;
+    const uint16_t *pv_base = prefix_page_table ? v_cache : prefix_v;
+#define PREFIX_ROW(j)                                                              \
+  (prefix_page_table                                                               \
+       ? (long)prefix_page_table[(long)d * max_prefix_pages + (j) / ORACLE_PAGE] * \
+                 ORACLE_PAGE + (j) % ORACLE_PAGE                                   \
+       : (long)prefix_cu[d] + (j))
+    int bad_page = 0;
+    if (prefix_page_table)
+      for (int pp = 0; pp * ORACLE_PAGE < P_b; ++pp) {
+        const int page = prefix_page_table[(long)d * max_prefix_pages + pp];
+        if (page < 0 || page >= num_pages) bad_page = 1;
+      }
+    if (bad_page) { bad = 1; continue; }
     const int L_b = branch_len[b];
     if (L_b < 0 || L_b > max_pages * ORACLE_PAGE) { bad = 1; continue; }
 
@@ -132,7 +158,7 @@ int oracle_branch_attn(const uint16_t *q, const uint16_t *prefix_k,
 
       /* visible prefix keys */
       for (int j = 0; j < P_b; ++j) {
-        const uint16_t *kv = prefix_k + ((long)(prefix_cu[d] + j) * H_kv + g) * D;
+        const uint16_t *kv = pk_base + (PREFIX_ROW(j) * H_kv + g) * D;
         double dot = 0.0;
         for (int c = 0; c < D; ++c) dot += bf16_to_double(qv[c]) * bf16_to_double(kv[c]);
         s[n++] = scale * dot;
@@ -162,7 +188,7 @@ int oracle_branch_attn(const uint16_t *q, const uint16_t *prefix_k,
       /* second walk over the same visible keys, in the same order */
       int t = 0;
       for (int j = 0; j < P_b; ++j, ++t) {
-        const uint16_t *vv = prefix_v + ((long)(prefix_cu[d] + j) * H_kv + g) * D;
+        const uint16_t *vv = pv_base + (PREFIX_ROW(j) * H_kv + g) * D;
         const double w = exp(s[t] - M) / denom;
         for (int c = 0; c < D; ++c) o[c] += w * bf16_to_double(vv[c]);
       }
@@ -178,6 +204,7 @@ int oracle_branch_attn(const uint16_t *q, const uint16_t *prefix_k,
       lse[row * H_q + h] = M + log(denom);
     }
     free(s);
+#undef PREFIX_ROW
   }
   return bad ? -1 : 0;
 }

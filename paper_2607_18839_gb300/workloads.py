@@ -73,6 +73,9 @@ class BranchDecodeInputs:
     page_table: np.ndarray    # int32 [B, max_pages]
     branch_len: np.ndarray    # int32 [B]
     branch_prefix_len: Optional[np.ndarray] = None  # int32 [B] or None
+    # paged prefix: page d's prefix token j is slot j % 16 of pool page
+    # prefix_page_table[d, j // 16]; int32 [n_docs, max_prefix_pages] or None
+    prefix_page_table: Optional[np.ndarray] = None
     scale: float = 0.0        # 0 -> 1/sqrt(D)
     name: str = "custom"
     meta: dict = field(default_factory=dict)
@@ -88,6 +91,10 @@ class BranchDecodeInputs:
     @property
     def max_prefix_len(self) -> int:
         return int(np.max(np.diff(self.prefix_cu))) if self.n_docs else 0
+
+    @property
+    def max_prefix_pages(self) -> int:
+        return 0 if self.prefix_page_table is None else int(self.prefix_page_table.shape[1])
 
 
 def _normal_bf16(rng: np.random.Generator, shape, std: float) -> np.ndarray:
@@ -172,6 +179,47 @@ def build_inputs(
         scale=scale, name=name,
         meta=dict(seed=seed, suffix_lens=suffix_lens.astype(np.int32)),
     )
+
+
+def page_the_prefix(inp: BranchDecodeInputs, seed: int, extra_pages: int = 0) -> BranchDecodeInputs:
+    """The same workload with every page's prefix moved into the KV pool.
+
+    Page d's prefix occupies ceil(P_d / 16) pool pages, placed with the
+    private pages in one seeded random physical order; slots past P_d in the
+    last prefix page hold unrelated finite values.  The contiguous
+    ``prefix_k`` / ``prefix_v`` are kept (same keys, for comparisons).
+    """
+    rng = np.random.default_rng(seed)
+    P = np.diff(inp.prefix_cu).astype(np.int64)
+    n_pp = (P + PAGE - 1) // PAGE
+    max_pp = int(max(1, n_pp.max() if len(n_pp) else 1))
+    n_new = int(n_pp.sum()) + extra_pages
+    total = inp.num_pages + n_new
+    perm = rng.permutation(total).astype(np.int32)
+    old_to_new = perm[:inp.num_pages]  # private page p moves to old_to_new[p]
+    k_cache = _normal_bf16(rng, (total, PAGE, inp.H_kv, inp.D), 0.5)
+    v_cache = _normal_bf16(rng, (total, PAGE, inp.H_kv, inp.D), 0.5)
+    k_cache[old_to_new] = inp.k_cache
+    v_cache[old_to_new] = inp.v_cache
+    ppt = rng.integers(0, total, size=(inp.n_docs, max_pp)).astype(np.int32)
+    cursor = inp.num_pages
+    for d in range(inp.n_docs):
+        base = int(inp.prefix_cu[d])
+        for pp in range(int(n_pp[d])):
+            pg = int(perm[cursor])
+            cursor += 1
+            ppt[d, pp] = pg
+            n = min(PAGE, int(P[d]) - pp * PAGE)
+            k_cache[pg, :n] = inp.prefix_k[base + pp * PAGE: base + pp * PAGE + n]
+            v_cache[pg, :n] = inp.prefix_v[base + pp * PAGE: base + pp * PAGE + n]
+    return BranchDecodeInputs(
+        n_docs=inp.n_docs, B=inp.B, m=inp.m, H_q=inp.H_q, H_kv=inp.H_kv, D=inp.D,
+        num_pages=total, max_pages=inp.max_pages, q=inp.q, prefix_k=inp.prefix_k,
+        prefix_v=inp.prefix_v, prefix_cu=inp.prefix_cu, branch_cu=inp.branch_cu,
+        k_cache=k_cache, v_cache=v_cache, page_table=old_to_new[inp.page_table],
+        branch_len=inp.branch_len, branch_prefix_len=inp.branch_prefix_len,
+        prefix_page_table=ppt, scale=inp.scale, name=inp.name + "-paged",
+        meta=dict(inp.meta, paged_prefix_seed=seed))
 
 
 def _lognormal_suffix(rng, n):

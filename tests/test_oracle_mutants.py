@@ -33,6 +33,11 @@ MUTATIONS = [
      "for (int j = 0; j < 0; ++j, ++t) {", False),
     ("max not subtracted in the weights", "const double w = exp(s[t] - M) / denom;",
      "const double w = exp(s[t]) / denom;", True),
+    ("paged prefix slot transposed",
+     "ORACLE_PAGE + (j) % ORACLE_PAGE ", "ORACLE_PAGE + ((j) / ORACLE_PAGE) % ORACLE_PAGE ", False),
+    ("paged prefix reads page 0's table row",
+     "prefix_page_table[(long)d * max_prefix_pages + (j) / ORACLE_PAGE]",
+     "prefix_page_table[(long)0 * max_prefix_pages + (j) / ORACLE_PAGE]", False),
     ("argmax keeps the last of equal maxima", "if (!seen || x > best_val) {",
      "if (!seen || x >= best_val) {", False),
     ("accepted length counts the bonus token", "accepted_len[b] = k;",
@@ -48,6 +53,8 @@ PIN_TESTS = [
     pins.test_gqa_groups_contiguous_query_heads,
     pins.test_no_visible_key_gives_zero_and_minus_inf,
     pins.test_causality_among_the_m_queries,
+    lambda: [pins.test_paged_prefix_matches_brute_force_on_the_same_keys(c) for c in range(6)],
+    pins.test_paged_prefix_follows_the_table,
     pins.test_accept_closed_forms,
     pins.test_accept_ties_lowest_index_and_nan_ignored,
     pins.test_accept_matches_numpy_argmax_brute_force,
@@ -67,7 +74,7 @@ def _bind(path):
     lib = ctypes.CDLL(path)
     P, I = ctypes.c_void_p, ctypes.c_int
     lib.oracle_branch_attn.restype = I
-    lib.oracle_branch_attn.argtypes = [P] * 10 + [I] * 8 + [ctypes.c_double, P, I, I, P, P]
+    lib.oracle_branch_attn.argtypes = [P] * 10 + [I] * 8 + [ctypes.c_double, P, I, I, P, P, P, I]
     lib.oracle_pmtp_accept.restype = None
     lib.oracle_pmtp_accept.argtypes = [P, P, I, I, I, P, P]
     lib.oracle_max_threads.restype = I

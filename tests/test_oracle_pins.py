@@ -312,3 +312,37 @@ def test_accept_matches_numpy_argmax_brute_force():
         while k < m and drafts[b, k] == ref_tok[b, k]:
             k += 1
         assert acc[b] == k
+
+
+@pytest.mark.parametrize("case", list(range(6)))
+def test_paged_prefix_matches_brute_force_on_the_same_keys(case):
+    # The prefix moved into the pool (own pages, random physical order, the
+    # contiguous buffers kept) must give the brute-force result over the
+    # contiguous keys; with the contiguous buffers wiped it must not change,
+    # so the paged mode reads the pool through the prefix page table.
+    inp = W.page_the_prefix(list(tiny_cases())[case], seed=70 + case, extra_pages=2)
+    bo, bl = brute_force(inp)
+    inp.prefix_k = np.full_like(inp.prefix_k, 0x7FC0)  # NaN bits: must never be read
+    inp.prefix_v = np.full_like(inp.prefix_v, 0x7FC0)
+    out, lse = oracle.branch_attn(inp)
+    assert np.array_equal(np.isinf(lse), np.isinf(bl))
+    fin = np.isfinite(bl)
+    np.testing.assert_allclose(lse[fin], bl[fin], rtol=0, atol=1e-12)
+    np.testing.assert_allclose(out, bo, rtol=0, atol=1e-12)
+
+
+def test_paged_prefix_follows_the_table():
+    # Swapping the first two prefix pages in the table moves keys across the
+    # fork limits (16 and 8: only page 0 visible), which changes what the
+    # branches see; swapping the pool pages back restores it exactly.
+    inp = W.page_the_prefix(W.build_inputs([40], [3], [4, 9, 20], 2, 4, 2, 8, seed=8,
+                                           branch_prefix_len=[16, 16, 8]), seed=9)
+    o0, _ = oracle.branch_attn(inp)
+    a, b = inp.prefix_page_table[0, 0], inp.prefix_page_table[0, 1]
+    inp.prefix_page_table[0, [0, 1]] = [b, a]
+    o1, _ = oracle.branch_attn(inp)
+    assert not np.allclose(o0, o1)
+    for cache in (inp.k_cache, inp.v_cache):
+        cache[[a, b]] = cache[[b, a]]
+    o2, _ = oracle.branch_attn(inp)
+    np.testing.assert_array_equal(o0, o2)
