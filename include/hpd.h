@@ -82,6 +82,11 @@ typedef enum {
  *   prefix keys  j <  P_b   (P_b = branch_prefix_len[b] if given, else P_d)
  *   private keys j <= L_b - m + i
  * Private key j is slot j % 16 of physical page page_table[b][j / 16].
+ * The prefix is contiguous (prefix_k / prefix_v rows), or, when
+ * prefix_page_table is set, paged in the same pool: prefix token j of page d
+ * is slot j % 16 of physical page prefix_page_table[d][j / 16], shared by all
+ * of the page's branches without a copy (Algorithm 1: a forked branch shares
+ * its parent's KV pages; Sec. 3.3).
  * S_j = scale * <q, k_j>; out = softmax(S) V over the visible keys;
  * lse = ln sum_j exp(S_j).  No visible key: out = 0, lse = -inf.
  */
@@ -111,6 +116,14 @@ typedef struct {
   void *workspace;          /* 256-byte aligned, initialised once by
                                hpd_workspace_init; one call at a time per workspace */
   size_t workspace_bytes;
+  /* Paged prefix (NULL: contiguous).  When set, prefix_k / prefix_v are not
+   * read (may be NULL), prefix_cu still gives every P_d (only its differences
+   * matter, bounded by prefix_tokens) and P_d <= 16 * max_prefix_pages, else
+   * HPD_DEVERR_PREFIX_CU and the prefix is cut there.  A table entry outside
+   * [0, num_pages) is flagged HPD_DEVERR_PAGE_ID and read as page 0; entries
+   * past a page's last prefix page are not read. */
+  const int32_t *prefix_page_table; /* [n_docs][max_prefix_pages]                 */
+  int max_prefix_pages;             /* >= 1 columns when prefix_page_table is set */
 } hpd_branch_attn_args;
 
 /* Bytes of workspace hpd_branch_attn needs for these host scalars (the

@@ -58,7 +58,7 @@ __global__ void __launch_bounds__(kThreads) attn_stage_kernel(const AttnParams p
 
   // ------------------------------------------------------ work decode --
   int g, slot, r0, nrows, tokbase, k_begin, k_end;
-  int pc0 = 0, bidx = 0, L = 0, P_d = 0;
+  int pc0 = 0, bidx = 0, L = 0, P_d = 0, doc = 0;
   if constexpr (PREFIX) {
     g = blockIdx.y;
     const int split = blockIdx.z;
@@ -100,11 +100,10 @@ __global__ void __launch_bounds__(kThreads) attn_stage_kernel(const AttnParams p
     const int d = s_info[0];
     if (d < 0) return;  // grid is an upper bound of the tile count
     const int lt = s_info[1], b0 = s_info[2], b1 = s_info[3];
-    int a0 = p.prefix_cu[d], a1 = p.prefix_cu[d + 1];
-    if (a0 < 0 || a1 < a0 || a1 > p.prefix_tokens) flag_error(p.err, HPD_DEVERR_PREFIX_CU);
-    pc0 = min(max(a0, 0), p.prefix_tokens);
-    const int pc1 = min(max(a1, pc0), p.prefix_tokens);
-    P_d = pc1 - pc0;
+    bool bad;
+    page_prefix(p, d, pc0, P_d, bad);
+    if (bad) flag_error(p.err, HPD_DEVERR_PREFIX_CU);
+    doc = d;
     const int R_d = (b1 - b0) * m * G;
     r0 = lt * TILE_M;
     nrows = min(TILE_M, R_d - r0);
@@ -187,10 +186,14 @@ __global__ void __launch_bounds__(kThreads) attn_stage_kernel(const AttnParams p
   }
 
   // --------------------------------------------------------- loaders --
-  const __nv_bfloat16 *Kbase = PREFIX ? p.prefix_k : p.k_cache;
-  const __nv_bfloat16 *Vbase = PREFIX ? p.prefix_v : p.v_cache;
+  const bool pool = !PREFIX || p.prefix_page_table;
+  const __nv_bfloat16 *Kbase = pool ? p.k_cache : p.prefix_k;
+  const __nv_bfloat16 *Vbase = pool ? p.v_cache : p.prefix_v;
   auto key_row = [&](int j) -> size_t {  // element offset of key j's head-g vector
     if constexpr (PREFIX) {
+      if (p.prefix_page_table)  // paged prefix: slot j % 16 of a pool page
+        return ((static_cast<size_t>(prefix_page(p, doc, j / kPage)) * kPage + (j % kPage)) *
+                    p.H_kv + g) * D;
       return (static_cast<size_t>(pc0 + j) * p.H_kv + g) * D;
     } else {
       int page = p.page_table[static_cast<size_t>(bidx) * p.max_pages + j / kPage];

@@ -12,9 +12,14 @@
 // branch: that is the shared-prefix KV reuse the method relies on.
 //
 // Key blocks: a unit walks 128-key blocks of two kinds,
-//   prefix blocks  128 consecutive prefix keys (3-D TMA box per 64 columns),
+//   prefix blocks  128 consecutive prefix keys: one 3-D TMA box per 64
+//                  columns from the contiguous prefix, or, with a paged
+//                  prefix, 8 pool pages of 16 keys from the page's prefix
+//                  page table (Algorithm 1: forks share the parent's pages),
 //   suffix blocks  8 pages of 16 keys, packed from the private caches of the
-//                  unit's branches in branch order (4-D TMA box per page).
+//                  unit's branches in branch order.
+// A paged block whose 8 pages are consecutive pool pages loads as one 8-page
+// 4-D box per 64 columns, else as one box per page.
 // For every row and block the visible columns form one interval [lo, hi):
 // a prefix block's keys below the row's limit, or the row's own branch's
 // pages up to its causal bound.  Rows of other branches see nothing of a
@@ -91,7 +96,8 @@ struct UnitMeta {
   int pc0;       // first prefix token of the page
   int blk_lo;    // first block of the split
   int n_blocks;  // blocks of the split (> 0)
-  int pad;
+  int doc;       // page (document) of the tile
+  int pp_last;   // paged prefix: last prefix page any row of the tile sees
   int page_start[kMaxUnitBranches + 1];  // packed page offset of each branch
   int blen[kMaxUnitBranches];            // private length L_b (clamped)
   int fork[kMaxUnitBranches];            // prefix keys visible to the branch
@@ -177,7 +183,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     branch_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k,
                           const __grid_constant__ CUtensorMap tm_v,
                           const __grid_constant__ CUtensorMap tm_kc,
-                          const __grid_constant__ CUtensorMap tm_vc, const AttnParams p) {
+                          const __grid_constant__ CUtensorMap tm_vc,
+                          const __grid_constant__ CUtensorMap tm_k8,
+                          const __grid_constant__ CUtensorMap tm_v8, const AttnParams p) {
   using L = TcLayout<D>;
   extern __shared__ uint8_t smem_raw[];
   __shared__ TcShared sh;
@@ -284,11 +292,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           base += __shfl_sync(0xffffffffu, incl, 31);
         }
         if (d < 0) continue;
-        const int a0 = p.prefix_cu[d], a1 = p.prefix_cu[d + 1];
-        if (lane == 0 && (a0 < 0 || a1 < a0 || a1 > p.prefix_tokens))
-          flag_error(p.err, HPD_DEVERR_PREFIX_CU);
-        const int pc0 = min(max(a0, 0), p.prefix_tokens);
-        const int P_d = min(max(a1, pc0), p.prefix_tokens) - pc0;
+        int pc0, P_d;
+        bool bad_prefix;
+        page_prefix(p, d, pc0, P_d, bad_prefix);
+        if (lane == 0 && bad_prefix) flag_error(p.err, HPD_DEVERR_PREFIX_CU);
         const int tok0 = b0 * m + lt * TT;
         const int ntok = min(TT, (b1 - b0) * m - lt * TT);
         const int b_lo = tok0 / m;
@@ -389,6 +396,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           M.nbc = nbc;
           M.nP = ceil_div_i(kmax, kBlk);
           M.pc0 = pc0;
+          M.doc = d;
+          M.pp_last = max(kmax - 1, 0) / kPage;
           M.blk_lo = blk_lo;
           M.n_blocks = blk_hi - blk_lo;
         }
@@ -411,6 +420,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&tm_v);
       prefetch_tmap(&tm_kc);
       prefetch_tmap(&tm_vc);
+      prefetch_tmap(&tm_k8);
+      prefetch_tmap(&tm_v8);
     }
     __syncwarp();
     int jbase = 0, issued_k = 0, issued_v = 0;
@@ -439,41 +450,64 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         return pg;
       };
-      // one block of K (or V) into stage `dst`
-      auto load_block = [&](int jb, uint32_t dst, uint32_t b, const CUtensorMap *prefix_map,
-                            const CUtensorMap *page_map) {
+      // paged prefix: lane i < 8 fetches the pool page of prefix page
+      // 8 jb + i (pages past the last one any row sees repeat it: finite
+      // values, never visible); called before waiting for the ring slot so
+      // the lookup overlaps the wait
+      const bool paged_prefix = p.prefix_page_table != nullptr;
+      auto prefix_pid = [&](int jb) -> int {
+        if (!paged_prefix || jb >= nP || lane >= kPagesPerBlock) return 0;
+        return prefix_page(p, M.doc, min(jb * kPagesPerBlock + lane, M.pp_last));
+      };
+      // one block of K (or V) into stage `dst`.  A paged block is 8 pages
+      // (lane i < 8 holds page i); when they are consecutive pool pages one
+      // 8-page box loads them all, else one box per page.
+      auto load_block = [&](int jb, int pid, uint32_t dst, uint32_t b,
+                            const CUtensorMap *prefix_map, const CUtensorMap *page_map,
+                            const CUtensorMap *run_map) {
         mbar_arrive_expect_tx_elect(b, L::kTileBytes);
-        if (jb < nP) {
+        if (jb < nP && !paged_prefix) {
           for (int c = 0; c < L::kChunks; ++c)
             tma_load_3d_elect(dst + c * L::kChunkBytes, prefix_map, b, c * 64, g, pc0 + jb * kBlk);
+          return;
+        }
+        int pg = pid;
+        if (jb >= nP && lane < kPagesPerBlock)  // slots past the last page repeat it
+          pg = page_of(min((jb - nP) * kPagesPerBlock + lane, P_s - 1));
+        const int next = __shfl_down_sync(0xffffffffu, pg, 1);
+        const unsigned run =
+            __ballot_sync(0xffffffffu, lane < kPagesPerBlock - 1 && next == pg + 1);
+        if (p.num_pages >= kPagesPerBlock && (run & 0x7fu) == 0x7fu) {
+          const int pg0 = __shfl_sync(0xffffffffu, pg, 0);
+          for (int c = 0; c < L::kChunks; ++c)
+            tma_load_4d_elect(dst + c * L::kChunkBytes, run_map, b, c * 64, g, 0, pg0);
         } else {
-          const int gp0 = (jb - nP) * kPagesPerBlock;
           for (int i = 0; i < kPagesPerBlock; ++i) {
-            // slots past the last page repeat it: finite values, never visible
-            const int pg = page_of(min(gp0 + i, P_s - 1));
+            const int pgi = __shfl_sync(0xffffffffu, pg, i);
             for (int c = 0; c < L::kChunks; ++c)
               tma_load_4d_elect(dst + c * L::kChunkBytes + i * kPage * 128, page_map, b, c * 64, g,
-                                0, pg);
+                                0, pgi);
           }
         }
       };
       for (int j = 0; j < nb; ++j) {
         const int jg = jbase + j;
+        const int pid = prefix_pid(blk_lo + j);
         if (is_k) {
           const int s = jg % L::kKStages;
           if (jg >= L::kKStages &&
               !(ok = wait_bar(sh.k_empty[s], ((jg / L::kKStages) - 1) & 1)))
             break;
-          load_block(blk_lo + j, sbase + L::kK + s * L::kTileBytes, bar(sh.k_full[s]), &tm_k,
-                     &tm_kc);
+          load_block(blk_lo + j, pid, sbase + L::kK + s * L::kTileBytes, bar(sh.k_full[s]), &tm_k,
+                     &tm_kc, &tm_k8);
           issued_k = jg + 1;
         } else {
           const int s = jg % L::kVStages;
           if (jg >= L::kVStages &&
               !(ok = wait_bar(sh.v_empty[s], ((jg / L::kVStages) - 1) & 1)))
             break;
-          load_block(blk_lo + j, sbase + L::kV + s * L::kTileBytes, bar(sh.v_full[s]), &tm_v,
-                     &tm_vc);
+          load_block(blk_lo + j, pid, sbase + L::kV + s * L::kTileBytes, bar(sh.v_full[s]), &tm_v,
+                     &tm_vc, &tm_v8);
           issued_v = jg + 1;
         }
       }
@@ -787,10 +821,13 @@ template <int D>
 cudaError_t launch_tc(const AttnParams &p, bool overlap, cudaStream_t s) {
   using L = TcLayout<D>;
   static_assert(L::kDynSmem + sizeof(TcShared) <= 227 * 1024, "shared memory");
-  CUtensorMap tk, tv, tkc, tvc;
+  CUtensorMap tk, tv, tkc, tvc, tk8, tv8;
   cudaError_t e = tc::make_prefix_maps(p, &tk, &tv);
   if (e == cudaSuccess) e = tc::make_page_map(&tkc, p.k_cache, D, p.H_kv, p.num_pages);
   if (e == cudaSuccess) e = tc::make_page_map(&tvc, p.v_cache, D, p.H_kv, p.num_pages);
+  const int run = std::min(kPagesPerBlock, p.num_pages);  // box never longer than the pool
+  if (e == cudaSuccess) e = tc::make_page_map(&tk8, p.k_cache, D, p.H_kv, p.num_pages, run);
+  if (e == cudaSuccess) e = tc::make_page_map(&tv8, p.v_cache, D, p.H_kv, p.num_pages, run);
   if (e != cudaSuccess) return e;
   static std::atomic<uint64_t> configured{0};
   int dev = 0;
@@ -812,7 +849,7 @@ cudaError_t launch_tc(const AttnParams &p, bool overlap, cudaStream_t s) {
   }
   const dim3 grid(static_cast<unsigned>(std::min(p.n_units, sms[dev & 63])), 1, 1);
   return launch_kernel(overlap, branch_attn_tc_kernel<D>, grid, dim3(kThreads), L::kDynSmem, s,
-                       tk, tv, tkc, tvc, p);
+                       tk, tv, tkc, tvc, tk8, tv8, p);
 }
 
 }  // namespace

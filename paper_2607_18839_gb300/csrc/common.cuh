@@ -46,6 +46,8 @@ struct AttnParams {
   const __nv_bfloat16 *v_cache;
   const int32_t *page_table;
   const int32_t *branch_len;
+  const int32_t *prefix_page_table;  // [n_docs][max_prefix_pages], or null: contiguous prefix
+  int max_prefix_pages;
   int n_docs, B, m, H_q, H_kv, G, D;
   int num_pages, max_pages, prefix_tokens;
   float scale_log2;  // softmax scale * log2(e)
@@ -64,6 +66,32 @@ struct AttnParams {
 // ------------------------------------------------------- device helpers --
 __device__ __forceinline__ void flag_error(uint32_t *err, uint32_t bit) {
   if (err) atomicOr(err, bit);
+}
+
+// Prefix of page d: its first token pc0 in the contiguous layout and its
+// length P_d, clamped to the buffers (and, paged, to the table width); bad
+// when prefix_cu is out of range (the caller flags HPD_DEVERR_PREFIX_CU).
+__device__ __forceinline__ void page_prefix(const AttnParams &p, int d, int &pc0, int &P_d,
+                                            bool &bad) {
+  const int a0 = p.prefix_cu[d], a1 = p.prefix_cu[d + 1];
+  bad = a0 < 0 || a1 < a0 || a1 > p.prefix_tokens;
+  pc0 = min(max(a0, 0), p.prefix_tokens);
+  P_d = min(max(a1, pc0), p.prefix_tokens) - pc0;
+  if (p.prefix_page_table && P_d > p.max_prefix_pages * kPage) {
+    bad = true;
+    P_d = p.max_prefix_pages * kPage;
+  }
+}
+
+// Pool page holding prefix page pp of page d (paged prefix); an id out of
+// range is flagged and replaced by page 0.
+__device__ __forceinline__ int prefix_page(const AttnParams &p, int d, int pp) {
+  int pg = p.prefix_page_table[static_cast<size_t>(d) * p.max_prefix_pages + pp];
+  if (pg < 0 || pg >= p.num_pages) {
+    flag_error(p.err, HPD_DEVERR_PAGE_ID);
+    pg = 0;
+  }
+  return pg;
 }
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {

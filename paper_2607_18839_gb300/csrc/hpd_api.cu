@@ -37,6 +37,7 @@ hpd_status check_scalars(const hpd_branch_attn_args *a) {
   if (a->n_docs < 1 || a->B < 1 || a->m < 1 || a->H_q < 1 || a->H_kv < 1 || a->num_pages < 1 ||
       a->max_pages_per_branch < 1 || a->prefix_tokens < 0 || a->max_prefix_len < 0)
     return HPD_ERR_INVALID_ARG;
+  if (a->prefix_page_table && a->max_prefix_pages < 1) return HPD_ERR_INVALID_ARG;
   if (a->m > 16) return HPD_ERR_UNSUPPORTED;
   if (a->H_q % a->H_kv != 0) return HPD_ERR_INVALID_ARG;
   if (a->H_q / a->H_kv > 16) return HPD_ERR_UNSUPPORTED;
@@ -53,8 +54,10 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
   hpd::Plan pl{};
   pl.G = a->H_q / a->H_kv;
   pl.rows_total = a->B * a->m;
-  const int maxP = a->max_prefix_len > 0 ? std::min(a->max_prefix_len, a->prefix_tokens)
-                                         : a->prefix_tokens;
+  int maxP = a->max_prefix_len > 0 ? std::min(a->max_prefix_len, a->prefix_tokens)
+                                   : a->prefix_tokens;
+  if (a->prefix_page_table)
+    maxP = static_cast<int>(std::min<long long>(maxP, 16LL * a->max_prefix_pages));
   pl.use_tc = (a->D == 64 || a->D == 128) && (kTcTileRows % pl.G == 0);
   if (pl.use_tc) {
     // tcgen05 kernel: units of 128 stacked rows (128 / G tokens) of one
@@ -174,12 +177,13 @@ hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t st
   if (!a->q || !a->prefix_cu || !a->branch_cu || !a->k_cache || !a->v_cache || !a->page_table ||
       !a->branch_len || !a->out)
     return HPD_ERR_INVALID_ARG;
-  if (a->prefix_tokens > 0 && (!a->prefix_k || !a->prefix_v)) return HPD_ERR_INVALID_ARG;
+  if (a->prefix_tokens > 0 && !a->prefix_page_table && (!a->prefix_k || !a->prefix_v))
+    return HPD_ERR_INVALID_ARG;
   if (!aligned(a->q, 16) || !aligned(a->prefix_k, 16) || !aligned(a->prefix_v, 16) ||
       !aligned(a->k_cache, 16) || !aligned(a->v_cache, 16) || !aligned(a->out, 16) ||
       !aligned(a->lse, 4) || !aligned(a->prefix_cu, 4) || !aligned(a->branch_cu, 4) ||
       !aligned(a->page_table, 4) || !aligned(a->branch_len, 4) ||
-      !aligned(a->branch_prefix_len, 4))
+      !aligned(a->branch_prefix_len, 4) || !aligned(a->prefix_page_table, 4))
     return HPD_ERR_INVALID_ARG;
   const hpd::Plan pl = make_plan(a);
   if (!a->workspace || !aligned(a->workspace, kAlign) || a->workspace_bytes < pl.bytes)
@@ -193,6 +197,8 @@ hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t st
   p.prefix_cu = a->prefix_cu;
   p.branch_cu = a->branch_cu;
   p.branch_prefix_len = a->branch_prefix_len;
+  p.prefix_page_table = a->prefix_page_table;
+  p.max_prefix_pages = a->prefix_page_table ? a->max_prefix_pages : 0;
   p.k_cache = static_cast<const __nv_bfloat16 *>(a->k_cache);
   p.v_cache = static_cast<const __nv_bfloat16 *>(a->v_cache);
   p.page_table = a->page_table;

@@ -166,16 +166,18 @@ inline cudaError_t make_map(CUtensorMap *map, const void *base, uint64_t d0, uin
 }
 
 // 4-D bf16 tensor map over the paged cache [pages][16][H_kv][D]: one box
-// is one page of one KV head (64 columns x 1 head x 16 tokens x 1 page).
+// is box_pages consecutive pages of one KV head (64 columns x 1 head x 16
+// tokens x box_pages pages), rows in page-then-slot order.
 inline cudaError_t make_page_map(CUtensorMap *map, const void *base, int D, int H_kv,
-                                 int num_pages) {
+                                 int num_pages, int box_pages = 1) {
   auto fn = encode_fn();
   if (!fn) return cudaErrorNotSupported;
   const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(H_kv),
                               static_cast<cuuint64_t>(kPage), static_cast<cuuint64_t>(num_pages)};
   const cuuint64_t row = static_cast<cuuint64_t>(D) * 2;
   const cuuint64_t strides[3] = {row, row * H_kv, row * H_kv * kPage};
-  const cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(kPage), 1};
+  const cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(kPage),
+                             static_cast<cuuint32_t>(box_pages)};
   const cuuint32_t es[4] = {1, 1, 1, 1};
   const CUresult r =
       fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides, box,
@@ -191,7 +193,7 @@ inline cudaError_t make_page_map(CUtensorMap *map, const void *base, int D, int 
 // no prefix at all (the maps are then never used).
 inline cudaError_t make_prefix_maps(const AttnParams &p, CUtensorMap *tk, CUtensorMap *tv) {
   const int D = p.D;
-  const bool has_prefix = p.prefix_tokens > 0;
+  const bool has_prefix = p.prefix_tokens > 0 && !p.prefix_page_table;  // paged: page maps
   const uint64_t T = has_prefix ? static_cast<uint64_t>(p.prefix_tokens) : 1;
   cudaError_t e = make_map(tk, has_prefix ? p.prefix_k : p.k_cache, D, p.H_kv, T, 64, 1, kBlk);
   if (e != cudaSuccess) return e;

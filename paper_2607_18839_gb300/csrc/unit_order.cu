@@ -80,10 +80,12 @@ __global__ void __launch_bounds__(kOrderThreads) unit_order_kernel(AttnParams p,
     if (d < nd) {
       const int c0 = min(max(p.branch_cu[d], 0), p.B);
       const int c1 = max(min(max(p.branch_cu[d + 1], 0), p.B), c0);
-      const int pc0 = min(max(p.prefix_cu[d], 0), p.prefix_tokens);
+      int pc0, P_d;
+      bool bad;
+      page_prefix(p, d, pc0, P_d, bad);
       c0s[d] = c0;
       c1s[d] = c1;
-      pds[d] = min(max(p.prefix_cu[d + 1], pc0), p.prefix_tokens) - pc0;
+      pds[d] = P_d;
       n = ceil_div_i((c1 - c0) * m, TT);
     }
     const int before = order_scan(n, ws, &run);

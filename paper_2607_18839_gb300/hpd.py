@@ -54,6 +54,7 @@ class hpd_branch_attn_args(ctypes.Structure):
         ("scale", ctypes.c_float),
         ("out", ctypes.c_void_p), ("lse", ctypes.c_void_p),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
+        ("prefix_page_table", ctypes.c_void_p), ("max_prefix_pages", ctypes.c_int),
     ]
 
 
@@ -251,14 +252,19 @@ class DeviceInputs:
     prefix_tokens: int
     max_prefix_len: int
     scale: float
+    prefix_page_table: "object" = None  # paged prefix: int32 [n_docs, max_prefix_pages]
+    max_prefix_pages: int = 0
 
     @staticmethod
     def from_host(inp, device="cuda", non_blocking=False) -> "DeviceInputs":
-        """Copy a ``workloads.BranchDecodeInputs`` to the device."""
+        """Copy a ``workloads.BranchDecodeInputs`` to the device (with a paged
+        prefix, the contiguous prefix buffers are not copied)."""
         import numpy as np
         import torch
 
         def bf(a):
+            if a is None:
+                return None
             t = torch.from_numpy(np.ascontiguousarray(a).view(np.int16))
             return t.to(device, non_blocking=non_blocking).view(torch.bfloat16)
 
@@ -266,15 +272,19 @@ class DeviceInputs:
             return None if a is None else torch.from_numpy(
                 np.ascontiguousarray(a, dtype=np.int32)).to(device, non_blocking=non_blocking)
 
+        ppt = getattr(inp, "prefix_page_table", None)
+        paged = ppt is not None
         return DeviceInputs(
-            q=bf(inp.q), prefix_k=bf(inp.prefix_k), prefix_v=bf(inp.prefix_v),
+            q=bf(inp.q), prefix_k=None if paged else bf(inp.prefix_k),
+            prefix_v=None if paged else bf(inp.prefix_v),
             prefix_cu=i32(inp.prefix_cu), branch_cu=i32(inp.branch_cu),
             branch_prefix_len=i32(inp.branch_prefix_len), k_cache=bf(inp.k_cache),
             v_cache=bf(inp.v_cache), page_table=i32(inp.page_table),
             branch_len=i32(inp.branch_len), n_docs=inp.n_docs, B=inp.B, m=inp.m, H_q=inp.H_q,
             H_kv=inp.H_kv, D=inp.D, num_pages=inp.num_pages, max_pages=inp.max_pages,
             prefix_tokens=inp.prefix_tokens, max_prefix_len=inp.max_prefix_len,
-            scale=float(inp.scale))
+            scale=float(inp.scale), prefix_page_table=i32(ppt),
+            max_prefix_pages=0 if ppt is None else int(ppt.shape[1]))
 
 
 def make_args(d: DeviceInputs, out=None, lse=None, workspace=None,
@@ -289,6 +299,8 @@ def make_args(d: DeviceInputs, out=None, lse=None, workspace=None,
     a.num_pages, a.max_pages_per_branch = d.num_pages, d.max_pages
     a.prefix_tokens, a.max_prefix_len = d.prefix_tokens, d.max_prefix_len
     a.scale = d.scale
+    a.prefix_page_table = _ptr(d.prefix_page_table)
+    a.max_prefix_pages = d.max_prefix_pages
     a.out, a.lse = _ptr(out), _ptr(lse)
     a.workspace = _ptr(workspace)
     a.workspace_bytes = int(workspace_bytes)

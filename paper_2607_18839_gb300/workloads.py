@@ -181,45 +181,63 @@ def build_inputs(
     )
 
 
-def page_the_prefix(inp: BranchDecodeInputs, seed: int, extra_pages: int = 0) -> BranchDecodeInputs:
+def page_the_prefix(inp: BranchDecodeInputs, seed: int, extra_pages: int = 0,
+                    runs: bool = False) -> BranchDecodeInputs:
     """The same workload with every page's prefix moved into the KV pool.
 
-    Page d's prefix occupies ceil(P_d / 16) pool pages, placed with the
-    private pages in one seeded random physical order; slots past P_d in the
-    last prefix page hold unrelated finite values.  The contiguous
-    ``prefix_k`` / ``prefix_v`` are kept (same keys, for comparisons).
+    Page d's prefix occupies ceil(P_d / 16) pool pages.  With ``runs`` they
+    are consecutive pool pages (one prefill allocation), the runs and the
+    private pages in a seeded random order; otherwise every page, prefix or
+    private, lands at a seeded random position.  Slots past P_d in the last
+    prefix page hold unrelated finite values.  The contiguous ``prefix_k`` /
+    ``prefix_v`` are kept (same keys, for comparisons).
     """
     rng = np.random.default_rng(seed)
     P = np.diff(inp.prefix_cu).astype(np.int64)
     n_pp = (P + PAGE - 1) // PAGE
     max_pp = int(max(1, n_pp.max() if len(n_pp) else 1))
-    n_new = int(n_pp.sum()) + extra_pages
-    total = inp.num_pages + n_new
-    perm = rng.permutation(total).astype(np.int32)
-    old_to_new = perm[:inp.num_pages]  # private page p moves to old_to_new[p]
+    total = inp.num_pages + int(n_pp.sum()) + extra_pages
+    # allocation units: each private page, each extra page, and each page's
+    # prefix (one unit of n_pp[d] pages with runs, else n_pp[d] units of one)
+    units = [("old", i, 1) for i in range(inp.num_pages)]
+    units += [("extra", i, 1) for i in range(extra_pages)]
+    for d in range(inp.n_docs):
+        if runs:
+            units.append(("pre", (d, 0), int(n_pp[d])))
+        else:
+            units += [("pre", (d, pp), 1) for pp in range(int(n_pp[d]))]
+    order = rng.permutation(len(units))
+    old_to_new = np.zeros(inp.num_pages, np.int32)
+    ppt = rng.integers(0, total, size=(inp.n_docs, max_pp)).astype(np.int32)
+    where = 0
+    for u in order:
+        kind, key, n = units[u]
+        if kind == "old":
+            old_to_new[key] = where
+        elif kind == "pre":
+            d, pp0 = key
+            ppt[d, pp0:pp0 + n] = np.arange(where, where + n, dtype=np.int32)
+        where += n
+    assert where == total
     k_cache = _normal_bf16(rng, (total, PAGE, inp.H_kv, inp.D), 0.5)
     v_cache = _normal_bf16(rng, (total, PAGE, inp.H_kv, inp.D), 0.5)
     k_cache[old_to_new] = inp.k_cache
     v_cache[old_to_new] = inp.v_cache
-    ppt = rng.integers(0, total, size=(inp.n_docs, max_pp)).astype(np.int32)
-    cursor = inp.num_pages
     for d in range(inp.n_docs):
         base = int(inp.prefix_cu[d])
         for pp in range(int(n_pp[d])):
-            pg = int(perm[cursor])
-            cursor += 1
-            ppt[d, pp] = pg
             n = min(PAGE, int(P[d]) - pp * PAGE)
-            k_cache[pg, :n] = inp.prefix_k[base + pp * PAGE: base + pp * PAGE + n]
-            v_cache[pg, :n] = inp.prefix_v[base + pp * PAGE: base + pp * PAGE + n]
+            k_cache[ppt[d, pp], :n] = inp.prefix_k[base + pp * PAGE: base + pp * PAGE + n]
+            v_cache[ppt[d, pp], :n] = inp.prefix_v[base + pp * PAGE: base + pp * PAGE + n]
     return BranchDecodeInputs(
         n_docs=inp.n_docs, B=inp.B, m=inp.m, H_q=inp.H_q, H_kv=inp.H_kv, D=inp.D,
         num_pages=total, max_pages=inp.max_pages, q=inp.q, prefix_k=inp.prefix_k,
         prefix_v=inp.prefix_v, prefix_cu=inp.prefix_cu, branch_cu=inp.branch_cu,
         k_cache=k_cache, v_cache=v_cache, page_table=old_to_new[inp.page_table],
         branch_len=inp.branch_len, branch_prefix_len=inp.branch_prefix_len,
-        prefix_page_table=ppt, scale=inp.scale, name=inp.name + "-paged",
-        meta=dict(inp.meta, paged_prefix_seed=seed))
+        prefix_page_table=ppt, scale=inp.scale,
+        name=inp.name + ("-paged-runs" if runs else "-paged"),
+        meta=dict(inp.meta, paged_prefix_seed=seed, paged_prefix_runs=runs))
 
 
 def _lognormal_suffix(rng, n):

@@ -40,9 +40,11 @@ def test_version_and_status_strings(lib):
 
 
 def test_struct_layout_matches_c():
-    # 10 pointers, 10 ints, a float, 3 pointers and a size_t (x86_64 / aarch64)
-    assert ctypes.sizeof(hpd.hpd_branch_attn_args) == 80 + 40 + 8 + 24 + 8
+    # 10 pointers, 10 ints, a float, 3 pointers, a size_t, a pointer and an
+    # int padded to 8 (x86_64 / aarch64)
+    assert ctypes.sizeof(hpd.hpd_branch_attn_args) == 80 + 40 + 8 + 24 + 8 + 8 + 8
     assert hpd.hpd_branch_attn_args.out.offset == 128
+    assert hpd.hpd_branch_attn_args.prefix_page_table.offset == 160
 
 
 def _args(**kw):
@@ -59,7 +61,7 @@ def test_workspace_size_rejects_bad_scalars(lib):
     assert hpd.hpd_branch_attn_workspace_size(_args()) > 0
     for bad in (dict(D=96), dict(H_q=15), dict(m=0), dict(m=17), dict(B=0), dict(n_docs=0),
                 dict(H_q=64, H_kv=2), dict(num_pages=0), dict(max_pages_per_branch=0),
-                dict(scale=float("nan"))):
+                dict(scale=float("nan")), dict(prefix_page_table=4096, max_prefix_pages=0)):
         assert hpd.hpd_branch_attn_workspace_size(_args(**bad)) == 0, bad
 
 
@@ -102,6 +104,8 @@ def test_struct_layouts_match_the_header(tmp_path):
         'int main(void) {\n'
         '  printf("%zu %zu %zu\\n", sizeof(hpd_branch_attn_args), offsetof(hpd_branch_attn_args, out),'
         ' offsetof(hpd_branch_attn_args, workspace_bytes));\n'
+        '  printf("%zu %zu\\n", offsetof(hpd_branch_attn_args, prefix_page_table),'
+        ' offsetof(hpd_branch_attn_args, max_prefix_pages));\n'
         '  printf("%zu %zu %zu\\n", sizeof(hpd_kv_args), offsetof(hpd_kv_args, workspace),'
         ' offsetof(hpd_kv_args, max_pages));\n'
         '  printf("%zu %zu %zu\\n", sizeof(hpd_fork_args), offsetof(hpd_fork_args, fork_token),'
@@ -113,5 +117,6 @@ def test_struct_layouts_match_the_header(tmp_path):
                                                               text=True, check=True).stdout.split("\n") if l]
     A, K, F = hpd.hpd_branch_attn_args, hpd.hpd_kv_args, hpd.hpd_fork_args
     assert got[0] == [ctypes.sizeof(A), A.out.offset, A.workspace_bytes.offset]
-    assert got[1] == [ctypes.sizeof(K), K.workspace.offset, K.max_pages.offset]
-    assert got[2] == [ctypes.sizeof(F), F.fork_token.offset, F.cap.offset]
+    assert got[1] == [A.prefix_page_table.offset, A.max_prefix_pages.offset]
+    assert got[2] == [ctypes.sizeof(K), K.workspace.offset, K.max_pages.offset]
+    assert got[3] == [ctypes.sizeof(F), F.fork_token.offset, F.cap.offset]

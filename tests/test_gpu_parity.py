@@ -119,6 +119,78 @@ def test_parity_full_size_sampled_branches(hpd, name):
     assert np.all(np.isfinite(lse)) and np.all(np.abs(out) <= 4.0)
 
 
+# ----------------------------------------------------------- paged prefix --
+
+@pytest.mark.parametrize("name", list(SMALL))
+def test_paged_prefix_small_elementwise(hpd, name):
+    # the prefix read through the page pool (contiguous buffers not passed)
+    inp = W.page_the_prefix(SMALL[name](), seed=90, extra_pages=3)
+    ref_out, ref_lse = oracle.branch_attn(inp)
+    out, lse, err = run_gpu(hpd, inp)
+    assert err == 0
+    compare(inp, out, lse, ref_out, ref_lse)
+
+
+@pytest.mark.parametrize("runs", [False, True])
+@pytest.mark.parametrize("name", ["c2", "c4", "g3_warp_mma_prefix", "many_pages_split_prefix"])
+def test_paged_prefix_equals_contiguous_bitwise(hpd, name, runs):
+    # same keys in the same blocks: the paged and contiguous layouts give
+    # identical bits (masked slots weigh exactly zero in both); with runs the
+    # prefix pages are consecutive in the pool and load as 8-page boxes
+    base = SMALL[name]() if name in SMALL else W.make_config(name)
+    o1, l1, e1 = run_gpu(hpd, base)
+    o2, l2, e2 = run_gpu(hpd, W.page_the_prefix(base, seed=91, runs=runs))
+    assert e1 == e2 == 0
+    np.testing.assert_array_equal(o1, o2)
+    np.testing.assert_array_equal(l1, l2)
+
+
+@pytest.mark.parametrize("runs", [False, True])
+@pytest.mark.parametrize("name", ["c3", "c4", "c5"])
+def test_paged_prefix_full_size_sampled_branches(hpd, name, runs):
+    inp = W.page_the_prefix(W.make_config(name), seed=92, runs=runs)
+    sel = np.array(sample_branches(inp), dtype=np.int32)
+    ref_out, ref_lse = oracle.branch_attn(inp, branch_sel=sel)
+    out, lse, err = run_gpu(hpd, inp)
+    assert err == 0
+    compare(inp, out, lse, ref_out, ref_lse, rows=branch_rows(inp, sel))
+
+
+def _defragment(inp):
+    """The same workload with each branch's private pages made consecutive
+    pool pages (in branch order), the unused pages after them."""
+    used = [int(p) for b in range(inp.B)
+            for p in inp.page_table[b, :(int(inp.branch_len[b]) + W.PAGE - 1) // W.PAGE]]
+    rest = [p for p in range(inp.num_pages) if p not in set(used)]
+    order = np.array(used + rest, np.int64)        # new id -> old id
+    new_of = np.empty(inp.num_pages, np.int32)
+    new_of[order] = np.arange(inp.num_pages, dtype=np.int32)
+    out = W.BranchDecodeInputs(**{**inp.__dict__})
+    out.k_cache, out.v_cache = inp.k_cache[order], inp.v_cache[order]
+    out.page_table = new_of[inp.page_table]
+    return out
+
+
+@pytest.mark.parametrize("name", ["c3", "long_suffix_splits"])
+def test_consecutive_private_pages_bitwise(hpd, name):
+    # private pages in consecutive pool pages load as 8-page boxes; the
+    # result is the same bits as with scattered pages
+    base = SMALL[name]() if name in SMALL else W.make_config(name)
+    o1, l1, e1 = run_gpu(hpd, base)
+    o2, l2, e2 = run_gpu(hpd, _defragment(base))
+    assert e1 == e2 == 0
+    np.testing.assert_array_equal(o1, o2)
+    np.testing.assert_array_equal(l1, l2)
+
+
+def test_paged_prefix_bad_page_id_is_flagged(hpd):
+    inp = W.page_the_prefix(W.build_inputs([100], [2], [3, 4], 2, 8, 2, 128, seed=45), seed=93)
+    inp.prefix_page_table[0, 1] = inp.num_pages + 5
+    out, lse, err = run_gpu(hpd, inp)
+    assert err & 0x8
+    assert np.all(np.isfinite(out))
+
+
 def test_c3_full_oracle_elementwise(hpd):
     inp = W.make_config("c3")
     ref_out, ref_lse = oracle.branch_attn(inp)
