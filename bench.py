@@ -2,10 +2,11 @@
 """Benchmark of the branch-decode step of Hierarchical Parallel Decoding.
 
 One step = one pass of the whole hot path over one batch of synthetic input:
-hpd_branch_attn (the tcgen05 shared-prefix stage, then the private-suffix
-stage over the paged KV, which also does the LSE merge) followed by
-hpd_pmtp_accept (greedy verification of the P-MTP
-drafts against bf16 logits over a 32,000-token vocabulary).
+hpd_branch_attn (one persistent tcgen05 kernel over every branch's shared
+prefix and paged private suffix, preceded by a unit-ordering pass when there
+are at least two units per SM and followed by the LSE merge of key splits
+when the keys are split) followed by hpd_pmtp_accept (greedy verification of
+the P-MTP drafts against bf16 logits over a 32,000-token vocabulary).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c2]
                     [--impl ours|reference]
@@ -443,6 +444,37 @@ def run_ours(args, world, rank, local):
                  "note": "hpd_fork_children over the step's branches (two launches); not part of "
                          "the step metric"}
 
+    # ---- the attention call on other layouts of the prefix and on the
+    # layout-branch workload (reported beside the step; one input replica)
+    def attn_call_us(inp_x):
+        op_x = H.BranchAttn(H.DeviceInputs.from_host(inp_x), stream)
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                op_x(stream)
+        torch.cuda.synchronize(dev)
+        g_x = capture(S, 0, lambda r, i: op_x(stream))
+        ms = timed(g_x, None, n_rep, sync_ranks=False) / (n_rep * S)
+        if op_x.errors(stream):
+            raise SystemExit(f"bench.py: error flags {op_x.errors(stream):#x} on {inp_x.name}")
+        return ms * 1e3, H.hpd_branch_attn_launches(op_x.args)
+
+    runs_us, _ = attn_call_us(W.page_the_prefix(inp, seed=7000 + cid, runs=True))
+    scat_us, _ = attn_call_us(W.page_the_prefix(inp, seed=7000 + cid, runs=False))
+    paged_line = {"us_per_call_consecutive_pages": runs_us, "us_per_call_scattered_pages": scat_us,
+                  "contiguous_us_per_call": attn_ms * 1e3,
+                  "note": "the same attention call with every page's prefix in the 16-token KV "
+                          "pool through a prefix page table: in consecutive pool pages (one "
+                          "prefill allocation) or scattered; one L2-warm input replica"}
+    lay = W.make_layout_config()
+    lay_us, lay_launch = attn_call_us(lay)
+    layout_line = {"workload": "8 pages, vision U[1024,3072], layout tokens U[64,512], each "
+                               "page's layout branch + U[4,24] content branches forked after "
+                               "a layout token (lognormal histories), m=4, Hq16/Hkv2, D128, "
+                               "paged prefix shared with the layout branch",
+                   "us_per_call": lay_us, "launches": lay_launch,
+                   "query_tokens_per_s": lay.B * lay.m / (lay_us * 1e-6),
+                   "note": "attention call only, one L2-warm input replica"}
+
     # ---- end to end: pinned host inputs in, results out, every step
     host_q = torch.from_numpy(inp.q.view(np.int16)).pin_memory()
     host_meta = [torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).pin_memory()
@@ -547,6 +579,8 @@ def run_ours(args, world, rank, local):
         "attn_call_us": attn_ms * 1e3,
         "kv_append_rollback": kv_line,
         "fork_children": fork_line,
+        "paged_prefix": paged_line,
+        "layout_branches": layout_line,
         "host_wall_ms_per_step": total_wall_ms / K,
         "cpu_baseline": cpu,
         "clocks": clk,

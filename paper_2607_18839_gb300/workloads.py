@@ -240,6 +240,129 @@ def page_the_prefix(inp: BranchDecodeInputs, seed: int, extra_pages: int = 0,
         meta=dict(inp.meta, paged_prefix_seed=seed, paged_prefix_runs=runs))
 
 
+def build_layout_inputs(
+    vision_lens,
+    layout_lens,
+    content_per_doc,
+    content_suffix,
+    m: int,
+    H_q: int,
+    H_kv: int,
+    D: int,
+    seed: int,
+    *,
+    std: float = 0.5,
+    extra_pages: int = 0,
+    name: str = "layout",
+) -> BranchDecodeInputs:
+    """One step in which every page's layout branch decodes beside the
+    content branches already forked from it (Sec. 3.3, Algorithm 1).
+
+    Page d's layout sequence is V_d vision tokens, then A_d layout tokens,
+    then the layout branch's m drafts of this step; it sits in one run of
+    consecutive pool pages (one allocation).  The shared prefix is
+    P_d = V_d + A_d (the prefix page table points into that run).  The
+    layout branch is branch ``branch_cu[d]``: an ordinary sequence with m
+    P-MTP queries whose context is only the page's own tokens, encoded with
+    no copy as fork prefix V16_d = 16 floor(V_d / 16) plus private pages =
+    the run's pages from V16_d on, L_b = P_d + m - V16_d (its drafts fill the
+    slots after P_d of the shared last prefix page, which no content branch
+    sees).  Content branch c forks after a layout token: fork prefix f_c
+    uniform in [V_d + 1, P_d] (V_d when A_d = 0), private history
+    content_suffix[c] + m in scattered pages.  ``meta['layout_seq_k']`` /
+    ``['layout_seq_v']`` hold each page's whole sequence (P_d + m tokens).
+    """
+    rng = np.random.default_rng(seed)
+    V = np.asarray(vision_lens, dtype=np.int64)
+    A = np.asarray(layout_lens, dtype=np.int64)
+    C = np.asarray(content_per_doc, dtype=np.int64)
+    n_docs = len(V)
+    assert len(A) == n_docs and len(C) == n_docs
+    P = V + A
+    B = int(n_docs + C.sum())
+    content_suffix = np.asarray(content_suffix, dtype=np.int64)
+    assert len(content_suffix) == int(C.sum())
+    run_pages = (P + m + PAGE - 1) // PAGE
+    content_len = (content_suffix + m).astype(np.int64)
+    content_pages = (content_len + PAGE - 1) // PAGE
+    total = int(run_pages.sum() + content_pages.sum()) + extra_pages
+    # allocation units: one run per page's layout sequence, one unit per
+    # content page (allocated over time), extra pages; random order
+    units = [("run", d, int(run_pages[d])) for d in range(n_docs)]
+    units += [("cpage", i, 1) for i in range(int(content_pages.sum()))]
+    units += [("extra", i, 1) for i in range(extra_pages)]
+    start = {}
+    where = 0
+    for u in rng.permutation(len(units)):
+        kind, key, n = units[u]
+        start[(kind, key)] = where
+        where += n
+    k_cache = _normal_bf16(rng, (total, PAGE, H_kv, D), std)
+    v_cache = _normal_bf16(rng, (total, PAGE, H_kv, D), std)
+
+    branch_cu = np.zeros(n_docs + 1, np.int32)
+    branch_cu[1:] = np.cumsum(C + 1)
+    prefix_cu = np.zeros(n_docs + 1, np.int32)
+    prefix_cu[1:] = np.cumsum(P)
+    V16 = (V // PAGE) * PAGE
+    branch_len = np.zeros(B, np.int32)
+    bpl = np.zeros(B, np.int32)
+    max_pages = int(max([run_pages[d] - V16[d] // PAGE for d in range(n_docs)] +
+                        ([int(content_pages.max())] if len(content_pages) else [1])))
+    page_table = rng.integers(0, total, size=(B, max_pages)).astype(np.int32)
+    max_pp = int(max(1, ((P + PAGE - 1) // PAGE).max()))
+    ppt = rng.integers(0, total, size=(n_docs, max_pp)).astype(np.int32)
+    seq_k, seq_v = [], []
+    prefix_k = np.zeros((int(P.sum()), H_kv, D), np.uint16)
+    prefix_v = np.zeros_like(prefix_k)
+    ci = 0
+    for d in range(n_docs):
+        r0 = start[("run", d)]
+        run = np.arange(r0, r0 + run_pages[d], dtype=np.int32)
+        n_seq = int(P[d] + m)
+        sk = k_cache[run].reshape(-1, H_kv, D)[:n_seq].copy()
+        sv = v_cache[run].reshape(-1, H_kv, D)[:n_seq].copy()
+        seq_k.append(sk)
+        seq_v.append(sv)
+        prefix_k[prefix_cu[d]:prefix_cu[d + 1]] = sk[:P[d]]
+        prefix_v[prefix_cu[d]:prefix_cu[d + 1]] = sv[:P[d]]
+        n_pp = int((P[d] + PAGE - 1) // PAGE)
+        ppt[d, :n_pp] = run[:n_pp]
+        b = int(branch_cu[d])  # the layout branch
+        bpl[b] = V16[d]
+        branch_len[b] = n_seq - V16[d]
+        own = run[V16[d] // PAGE:]
+        page_table[b, :len(own)] = own
+        for c in range(int(C[d])):
+            b = int(branch_cu[d]) + 1 + c
+            bpl[b] = int(rng.integers(V[d] + 1, P[d] + 1)) if A[d] > 0 else int(V[d])
+            branch_len[b] = content_len[ci]
+            for j in range(int(content_pages[ci])):
+                page_table[b, j] = start[("cpage", int(content_pages[:ci].sum()) + j)]
+            ci += 1
+    q = _normal_bf16(rng, (B * m, H_q, D), std)
+    return BranchDecodeInputs(
+        n_docs=n_docs, B=B, m=m, H_q=H_q, H_kv=H_kv, D=D, num_pages=total,
+        max_pages=max_pages, q=q, prefix_k=prefix_k, prefix_v=prefix_v, prefix_cu=prefix_cu,
+        branch_cu=branch_cu, k_cache=k_cache, v_cache=v_cache, page_table=page_table,
+        branch_len=branch_len, branch_prefix_len=bpl, prefix_page_table=ppt, name=name,
+        meta=dict(seed=seed, layout_branches=branch_cu[:-1].copy(), vision_lens=V.astype(np.int32),
+                  layout_lens=A.astype(np.int32), layout_seq_k=seq_k, layout_seq_v=seq_v))
+
+
+def make_layout_config(seed: int = 1006) -> BranchDecodeInputs:
+    """Layout-branch workload: 8 pages, vision U[1024, 3072] tokens, layout
+    tokens so far U[64, 512], U[4, 24] content branches per page forked
+    after a layout token with lognormal(4.5, 0.8) private histories, m=4,
+    H_q 16 / H_kv 2, D 128 (the shapes of the 32-page preset)."""
+    rng = np.random.default_rng(seed + 7919)
+    V = rng.integers(1024, 3073, size=8)
+    A = rng.integers(64, 513, size=8)
+    C = rng.integers(4, 25, size=8)
+    s = _lognormal_suffix(rng, int(C.sum()))
+    return build_layout_inputs(V, A, C, s, 4, 16, 2, 128, seed, name="layout")
+
+
 def _lognormal_suffix(rng, n):
     return np.clip(np.round(rng.lognormal(4.5, 0.8, size=n)), 1, 1024).astype(np.int64)
 
