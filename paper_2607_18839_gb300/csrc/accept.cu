@@ -38,6 +38,14 @@ __device__ __forceinline__ void consider(ArgBest &b, float x, int i) {
     b.i = i;
   }
 }
+// The same for a thread's own scan, whose indices only grow: a later equal
+// value never wins, so the strict comparison suffices.
+__device__ __forceinline__ void consider_next(ArgBest &b, float x, int i) {
+  if (x > b.v) {
+    b.v = x;
+    b.i = i;
+  }
+}
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
@@ -51,7 +59,8 @@ __device__ __forceinline__ int row_argmax(const __nv_bfloat16 *row, int V, float
   const int head = min(V, static_cast<int>(((16u - (addr & 15u)) & 15u) >> 1));
   const int nvec = (V - head) >> 3;
   const int tail = head + (nvec << 3);
-  for (int i = tid; i < head; i += kAcceptThreads) consider(best, __bfloat162float(row[i]), i);
+  // each thread visits its indices in increasing order: head, vectors, tail
+  for (int i = tid; i < head; i += kAcceptThreads) consider_next(best, __bfloat162float(row[i]), i);
   const uint4 *vrow = reinterpret_cast<const uint4 *>(row + head);
   for (int v0 = tid; v0 < nvec; v0 += kAcceptThreads * kAcceptUnroll) {
     uint4 x[kAcceptUnroll];
@@ -65,18 +74,19 @@ __device__ __forceinline__ int row_argmax(const __nv_bfloat16 *row, int V, float
       const int v = v0 + u * kAcceptThreads;
       if (v < nvec) {
         const int i0 = head + (v << 3);
-        consider(best, bf16_lo(x[u].x), i0 + 0);
-        consider(best, bf16_hi(x[u].x), i0 + 1);
-        consider(best, bf16_lo(x[u].y), i0 + 2);
-        consider(best, bf16_hi(x[u].y), i0 + 3);
-        consider(best, bf16_lo(x[u].z), i0 + 4);
-        consider(best, bf16_hi(x[u].z), i0 + 5);
-        consider(best, bf16_lo(x[u].w), i0 + 6);
-        consider(best, bf16_hi(x[u].w), i0 + 7);
+        consider_next(best, bf16_lo(x[u].x), i0 + 0);
+        consider_next(best, bf16_hi(x[u].x), i0 + 1);
+        consider_next(best, bf16_lo(x[u].y), i0 + 2);
+        consider_next(best, bf16_hi(x[u].y), i0 + 3);
+        consider_next(best, bf16_lo(x[u].z), i0 + 4);
+        consider_next(best, bf16_hi(x[u].z), i0 + 5);
+        consider_next(best, bf16_lo(x[u].w), i0 + 6);
+        consider_next(best, bf16_hi(x[u].w), i0 + 7);
       }
     }
   }
-  for (int i = tail + tid; i < V; i += kAcceptThreads) consider(best, __bfloat162float(row[i]), i);
+  for (int i = tail + tid; i < V; i += kAcceptThreads)
+    consider_next(best, __bfloat162float(row[i]), i);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float ov = __shfl_xor_sync(0xffffffffu, best.v, o);
