@@ -99,27 +99,39 @@ def algorithmic_work(inp, V=VOCAB):
     return per, dict(bytes=step_bytes, flops=prefix_flops + suffix_flops)
 
 
-def kernel_source_hash():
+# Sources each kernel is compiled from (its .cu, the headers it includes and
+# the host planner that shapes its launch): its recorded DRAM traffic stays
+# valid while these are unchanged.
+KERNEL_SOURCES = {
+    "branch_attn_tc": ["branch_attn_tc.cu", "tc_common.cuh", "sm100.cuh", "common.cuh", "hpd_api.cu"],
+    "unit_order": ["unit_order.cu", "common.cuh", "hpd_api.cu"],
+    "merge_splits": ["merge.cu", "common.cuh", "hpd_api.cu"],
+    "pmtp_accept": ["accept.cu", "common.cuh"],
+}
+
+
+def kernel_source_hash(kernel):
     h = hashlib.sha256()
-    for p in sorted(glob.glob(os.path.join(ROOT, "paper_2607_18839_gb300", "csrc", "*"))):
-        with open(p, "rb") as f:
-            h.update(os.path.basename(p).encode())
+    for name in KERNEL_SOURCES.get(kernel, []) + ["../../include/hpd.h"]:
+        with open(os.path.join(ROOT, "paper_2607_18839_gb300", "csrc", name), "rb") as f:
+            h.update(os.path.basename(name).encode())
             h.update(f.read())
     return h.hexdigest()[:16]
 
 
 def ncu_traffic(workload, kernel):
     """DRAM bytes per launch of `kernel` from the committed ncu summary, or
-    None when there is none or the kernels changed since it was taken."""
+    None when there is none or the kernel's sources changed since it was
+    taken."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
         t = json.load(f)
-    if t.get("kernel_source_hash") != kernel_source_hash():
-        return None
     e = t.get("workloads", {}).get(workload, {}).get(kernel)
-    return None if e is None else float(e["dram_bytes_per_launch"])
+    if e is None or e.get("source_hash") != kernel_source_hash(kernel):
+        return None
+    return float(e["dram_bytes_per_launch"])
 
 
 class ClockSampler:
