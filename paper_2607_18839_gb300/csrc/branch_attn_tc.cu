@@ -760,22 +760,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld_wait();
         if (!cur.valid) continue;
         const int dc = h * (D / 2) + c;  // output column
+        // 32-byte stores: each fills a whole sector of its row
         if (final_out) {
-          uint4 *dst = reinterpret_cast<uint4 *>(p.out + cur.pair * D + dc);
+          uint32_t w[16];
 #pragma unroll
-          for (int e = 0; e < 32; e += 8)
-            dst[e / 8] = make_uint4(
-                pack_bf16x2(__uint_as_float(o[e]) * inv, __uint_as_float(o[e + 1]) * inv),
-                pack_bf16x2(__uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv),
-                pack_bf16x2(__uint_as_float(o[e + 4]) * inv, __uint_as_float(o[e + 5]) * inv),
-                pack_bf16x2(__uint_as_float(o[e + 6]) * inv, __uint_as_float(o[e + 7]) * inv));
+          for (int e = 0; e < 16; ++e)
+            w[e] = pack_bf16x2(__uint_as_float(o[2 * e]) * inv, __uint_as_float(o[2 * e + 1]) * inv);
+          __nv_bfloat16 *dst = p.out + cur.pair * D + dc;
+          if (p.out_align32) {
+            st_global_v8(dst, w);
+            st_global_v8(dst + 16, w + 8);
+          } else {
+#pragma unroll
+            for (int e = 0; e < 16; e += 4)
+              reinterpret_cast<uint4 *>(dst)[e / 4] = make_uint4(w[e], w[e + 1], w[e + 2], w[e + 3]);
+          }
         } else {
           float *dst = p.o_part + slot_pair * D + dc;
 #pragma unroll
-          for (int e = 0; e < 32; e += 4)
-            *reinterpret_cast<float4 *>(dst + e) =
-                make_float4(__uint_as_float(o[e]) * inv, __uint_as_float(o[e + 1]) * inv,
-                            __uint_as_float(o[e + 2]) * inv, __uint_as_float(o[e + 3]) * inv);
+          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * inv);
+#pragma unroll
+          for (int e = 0; e < 32; e += 8) st_global_v8(dst + e, o + e);
         }
       }
       if (cur.valid && h == 0) {

@@ -60,6 +60,7 @@ struct AttnParams {
   int n_units;          // work units of the tcgen05 kernel (row tile x KV head x split)
   const int *unit_order;  // the order in which to take them (null: index order)
   __nv_bfloat16 *out;   // final output, written by the suffix stage
+  bool out_align32;     // out is 32-byte aligned (256-bit stores)
   float *lse;           // final lse (may be null)
 };
 
@@ -92,6 +93,13 @@ __device__ __forceinline__ int prefix_page(const AttnParams &p, int d, int pp) {
     pg = 0;
   }
   return pg;
+}
+
+// 256-bit global store of eight 32-bit words (32-byte aligned address).
+__device__ __forceinline__ void st_global_v8(void *p, const uint32_t *w) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(w[0]),
+               "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+               : "memory");
 }
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {

@@ -226,6 +226,7 @@ hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t st
   p.n_units = pl.tiles_max * a->H_kv * pl.S_p;
   p.unit_order = pl.lpt ? reinterpret_cast<int *>(ws + pl.off_order) : nullptr;
   p.out = static_cast<__nv_bfloat16 *>(a->out);
+  p.out_align32 = aligned(a->out, 32);
   p.lse = a->lse;
 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

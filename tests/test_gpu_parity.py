@@ -242,6 +242,25 @@ def test_marked_call_outside_and_inside_capture(hpd, name):
     assert ev[0].elapsed_time(ev[n]) > 0
 
 
+@pytest.mark.parametrize("name", ["c1", "multi_page_ragged", "c2"])
+def test_output_only_16_byte_aligned(hpd, name):
+    # the ABI asks 16-byte alignment of out; the kernel's 32-byte stores are
+    # used only when out allows them
+    inp = SMALL[name]()
+    d = hpd.DeviceInputs.from_host(inp)
+    op = hpd.BranchAttn(d)
+    ref = op()[0].clone()
+    n = ref.numel()
+    big = torch.zeros(n + 8, dtype=torch.bfloat16, device=ref.device)
+    out16 = big[8:].view(ref.shape)  # 16 bytes past a 256-byte boundary
+    assert out16.data_ptr() % 32 == 16
+    args = hpd.make_args(d, out16, op.lse, op.workspace, op.workspace.numel())
+    hpd.hpd_branch_attn(args, hpd._stream_handle(None))
+    torch.cuda.synchronize()
+    assert op.errors() == 0
+    assert torch.equal(out16, ref)
+
+
 def test_out_of_range_device_data_is_clamped_and_flagged(hpd):
     inp = W.build_inputs([40], [2], [20, 30], 2, 8, 2, 64, seed=39)
     inp.page_table[1, 0] = inp.num_pages + 5   # page id out of range
