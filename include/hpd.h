@@ -48,7 +48,7 @@ typedef struct CUstream_st *hpd_stream_t; /* identical to cudaStream_t */
 typedef enum {
   HPD_OK = 0,
   HPD_ERR_INVALID_ARG = 1, /* a host scalar or pointer is out of contract */
-  HPD_ERR_UNSUPPORTED = 2, /* a legal shape this build has no kernel for */
+  HPD_ERR_UNSUPPORTED = 2, /* a legal shape the library has no kernel for */
   HPD_ERR_WORKSPACE = 3,   /* workspace missing, misaligned or too small */
   HPD_ERR_CUDA = 4,        /* a CUDA runtime call or launch failed */
   HPD_ERR_TIMEOUT = 5      /* a bounded device-side wait gave up */
@@ -89,6 +89,11 @@ typedef enum {
  * its parent's KV pages; Sec. 3.3).
  * S_j = scale * <q, k_j>; out = softmax(S) V over the visible keys;
  * lse = ln sum_j exp(S_j).  No visible key: out = 0, lse = -inf.
+ *
+ * Alignment: q, prefix_k, prefix_v, k_cache, v_cache and out 16-byte aligned
+ * (a 32-byte aligned out is written with 32-byte stores), lse and the int32
+ * arrays 4-byte aligned, workspace 256-byte aligned; otherwise
+ * HPD_ERR_INVALID_ARG (HPD_ERR_WORKSPACE for the workspace).
  */
 typedef struct {
   const void *q;        /* bf16 [B*m][H_q][D]; row b*m + i                        */
@@ -143,8 +148,10 @@ hpd_status hpd_branch_attn(const hpd_branch_attn_args *args, hpd_stream_t stream
 
 /* Number of kernels one hpd_branch_attn call launches for these scalars
  * (0 if they are invalid).  When H_q / H_kv divides 128 the step runs on
- * tcgen05 tensor cores: one kernel for the shared prefix and the private
- * suffixes, plus a merge kernel when the keys are split across CTAs.
+ * tcgen05 tensor cores: one persistent kernel for the shared prefix and the
+ * private suffixes, preceded by a one-CTA pass that orders its work units
+ * longest first when there are at least two units per SM, and followed by a
+ * merge kernel when the keys are split across CTAs.
  * Otherwise: a warp-MMA shared-prefix kernel, then a warp-MMA private-suffix
  * kernel that also merges and writes out / lse. */
 int hpd_branch_attn_launches(const hpd_branch_attn_args *args);
