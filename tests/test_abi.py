@@ -120,3 +120,37 @@ def test_struct_layouts_match_the_header(tmp_path):
     assert got[1] == [A.prefix_page_table.offset, A.max_prefix_pages.offset]
     assert got[2] == [ctypes.sizeof(K), K.workspace.offset, K.max_pages.offset]
     assert got[3] == [ctypes.sizeof(F), F.fork_token.offset, F.cap.offset]
+
+
+def _workload_args(inp):
+    a = hpd.hpd_branch_attn_args()
+    for k, v in dict(n_docs=inp.n_docs, B=inp.B, m=inp.m, H_q=inp.H_q, H_kv=inp.H_kv, D=inp.D,
+                     num_pages=inp.num_pages, max_pages_per_branch=inp.max_pages,
+                     prefix_tokens=inp.prefix_tokens, max_prefix_len=inp.max_prefix_len,
+                     scale=inp.scale).items():
+        setattr(a, k, v)
+    return a
+
+
+def test_launch_plan_of_the_workloads(lib):
+    # host-only planning: which kernels one call launches (no GPU needed)
+    from paper_2607_18839_gb300 import workloads as W
+    expect = {
+        "c1": ["branch_attn_tc"],                        # one wave, no key split
+        "c2": ["branch_attn_tc", "merge_splits"],        # few tiles: keys split, then merged
+        "c4": ["unit_order", "branch_attn_tc"],          # >= 2 units per SM: longest first
+        "c5": ["branch_attn_tc"],
+    }
+    for name, kernels in expect.items():
+        a = _workload_args(W.make_config(name))
+        n = hpd.hpd_branch_attn_launches(a)
+        got = [hpd.hpd_branch_attn_kernel_name(a, k) for k in range(n)]
+        assert got == kernels, (name, got)
+        assert hpd.hpd_branch_attn_kernel_name(a, n) is None
+    # head ratios that do not divide 128 take the warp-MMA stages
+    g3 = W.build_inputs([200], [3], [4, 0, 33], 3, 6, 2, 128, seed=1)
+    a = _workload_args(g3)
+    assert [hpd.hpd_branch_attn_kernel_name(a, k) for k in range(2)] == ["prefix_stage",
+                                                                        "suffix_merge"]
+    # the unit order lives in the workspace: it grows with the units
+    assert hpd.hpd_branch_attn_workspace_size(_workload_args(W.make_config("c4"))) > 0
