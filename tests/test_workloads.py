@@ -45,3 +45,60 @@ def test_mix_drafts_rate():
     d = W.mix_drafts(t, 32000, 0.7, seed=3)
     rate = np.mean(d == t)
     assert 0.68 < rate < 0.72
+
+
+def _used_private_pages(inp):
+    out = {}
+    for b in range(inp.B):
+        n = (int(inp.branch_len[b]) + W.PAGE - 1) // W.PAGE
+        out[b] = inp.page_table[b, :n].tolist()
+    return out
+
+
+@pytest.mark.parametrize("runs", [False, True])
+def test_page_the_prefix_layout(runs):
+    base = W.build_inputs([40, 0, 33], [2, 1, 3], [5, 20, 1, 17, 40, 9], 2, 8, 2, 64, seed=3)
+    inp = W.page_the_prefix(base, seed=4, extra_pages=3, runs=runs)
+    assert inp.num_pages == base.num_pages + 3 + sum((int(p) + 15) // 16 for p in np.diff(base.prefix_cu))
+    priv = [pg for pages in _used_private_pages(inp).values() for pg in pages]
+    pre = []
+    for d in range(inp.n_docs):
+        P = int(inp.prefix_cu[d + 1] - inp.prefix_cu[d])
+        pages = inp.prefix_page_table[d, :(P + 15) // 16].tolist()
+        pre.extend(pages)
+        if runs and pages:  # one allocation: consecutive pool pages
+            assert pages == list(range(pages[0], pages[0] + len(pages)))
+        # the pool pages hold the prefix keys, slot by slot
+        for j in range(P):
+            assert np.array_equal(inp.k_cache[pages[j // 16], j % 16],
+                                  base.prefix_k[int(base.prefix_cu[d]) + j])
+    every = priv + pre
+    assert len(every) == len(set(every)) and all(0 <= x < inp.num_pages for x in every)
+    # the private keys moved with their pages
+    for b, pages in _used_private_pages(inp).items():
+        old = _used_private_pages(base)[b]
+        for a, o in zip(pages, old):
+            assert np.array_equal(inp.k_cache[a], base.k_cache[o])
+
+
+def test_layout_inputs_share_the_prefix_pages_without_copy():
+    inp = W.build_layout_inputs([37, 64, 16], [20, 0, 45], [2, 3, 0], [5, 17, 1, 40, 9], 3, 4, 2,
+                                64, seed=3)
+    V, A = inp.meta["vision_lens"], inp.meta["layout_lens"]
+    lay = inp.meta["layout_branches"]
+    priv = _used_private_pages(inp)
+    content_pages = [pg for b, pages in priv.items() if b not in set(lay.tolist()) for pg in pages]
+    assert len(content_pages) == len(set(content_pages))
+    for d in range(inp.n_docs):
+        P = int(V[d] + A[d])
+        b = int(lay[d])
+        pre = inp.prefix_page_table[d, :(P + 15) // 16].tolist()
+        own = priv[b]
+        v16 = int(V[d]) // 16
+        # the layout branch's private pages continue the prefix pages from the vision boundary
+        assert own[:len(pre) - v16] == pre[v16:]
+        assert not set(own) & set(content_pages)
+        # its sequence: prefix keys, then the drafts in the slots after P
+        seq = inp.meta["layout_seq_k"][d]
+        assert seq.shape[0] == P + inp.m
+        assert np.array_equal(inp.prefix_k[inp.prefix_cu[d]:inp.prefix_cu[d + 1]], seq[:P])
