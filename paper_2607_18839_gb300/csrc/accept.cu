@@ -51,7 +51,9 @@ __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w 
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
 // Argmax of one row of V bf16 values, reduced over the CTA (valid in thread 0).
-__device__ __forceinline__ int row_argmax(const __nv_bfloat16 *row, int V, float *s_v, int *s_i) {
+// s_none: a shared word, set when no value above -inf was found.
+__device__ __forceinline__ int row_argmax(const __nv_bfloat16 *row, int V, float *s_v, int *s_i,
+                                          int *s_none) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const float NEG_INF = -__int_as_float(0x7f800000);
   ArgBest best{NEG_INF, INT_MAX};
@@ -107,8 +109,22 @@ __device__ __forceinline__ int row_argmax(const __nv_bfloat16 *row, int V, float
       const int oi = __shfl_xor_sync(0xffffffffu, best.i, o);
       consider(best, ov, oi);
     }
+    if (lane == 0) *s_none = best.i == INT_MAX ? INT_MAX : -1;
   }
   __syncthreads();  // s_v / s_i are reused by the next row
+  if (*s_none == INT_MAX) {
+    // No value above -inf (the strict scan never takes a -inf): the maximum
+    // is -inf if the row holds one, at its first position (rare path).
+    __syncthreads();  // every thread has read the word before it is reused
+    for (int i = tid; i < V; i += kAcceptThreads)
+      if (__bfloat162float(row[i]) == NEG_INF) {
+        atomicMin(s_none, i);
+        break;
+      }
+    __syncthreads();
+    best.i = *s_none;
+    __syncthreads();  // read before the next row's flag
+  }
   return best.i == INT_MAX ? 0 : best.i;
 }
 
@@ -120,13 +136,14 @@ __global__ void __launch_bounds__(kAcceptThreads)
   __shared__ float s_v[kAcceptThreads / 32];
   __shared__ int s_i[kAcceptThreads / 32];
   __shared__ int s_tok[kMaxRows];  // used in the leader CTA
+  __shared__ int s_none;
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
   const int cs = static_cast<int>(cluster.num_blocks());
   const int b = blockIdx.x / cs;
   int *leader_tok = cluster.map_shared_rank(s_tok, 0);
   for (int j = rank; j < m; j += cs) {
-    const int tok = row_argmax(logits + (static_cast<size_t>(b) * m + j) * V, V, s_v, s_i);
+    const int tok = row_argmax(logits + (static_cast<size_t>(b) * m + j) * V, V, s_v, s_i, &s_none);
     if (threadIdx.x == 0) {
       out_tokens[static_cast<size_t>(b) * m + j] = tok;
       leader_tok[j] = tok;

@@ -299,6 +299,10 @@ def test_accept_ragged_vocab_ties_and_nan(hpd, V):
     vals[0, 0, :] = np.nan
     vals[1, 1, V // 2] = np.nan
     vals[2, 2, :] = -np.inf
+    vals[3, 3, :] = -np.inf             # the maximum is -inf, first after a run of NaN
+    vals[3, 3, :(V + 2) // 3] = np.nan
+    vals[4, 4, :] = np.nan              # a single -inf at the end
+    vals[4, 4, V - 1] = -np.inf
     logits = W.f32_to_bf16_bits(vals)
     ref_tok0, _ = oracle.pmtp_accept(logits, np.zeros((B, m), np.int32))
     drafts = W.mix_drafts(ref_tok0, V, 0.8, seed=V + 1)
