@@ -183,6 +183,16 @@ def test_consecutive_private_pages_bitwise(hpd, name):
     np.testing.assert_array_equal(l1, l2)
 
 
+def test_paged_prefix_table_too_narrow_is_flagged(hpd):
+    # a prefix page table with fewer columns than the page's prefix needs:
+    # the prefix is cut at the table's end and HPD_DEVERR_PREFIX_CU is set
+    inp = W.page_the_prefix(W.build_inputs([100], [2], [3, 4], 2, 8, 2, 128, seed=46), seed=94)
+    inp.prefix_page_table = np.ascontiguousarray(inp.prefix_page_table[:, :4])  # 64 of 100 tokens
+    out, lse, err = run_gpu(hpd, inp)
+    assert err & 0x1
+    assert np.all(np.isfinite(out)) and np.all(np.isfinite(lse))
+
+
 def test_paged_prefix_bad_page_id_is_flagged(hpd):
     inp = W.page_the_prefix(W.build_inputs([100], [2], [3, 4], 2, 8, 2, 128, seed=45), seed=93)
     inp.prefix_page_table[0, 1] = inp.num_pages + 5
@@ -310,6 +320,26 @@ def test_accept_ragged_vocab_ties_and_nan(hpd, V):
     tok, acc = run_accept(hpd, logits, drafts)
     np.testing.assert_array_equal(tok, ref_tok)
     np.testing.assert_array_equal(acc, ref_acc)
+
+
+def test_accept_more_rows_than_the_cluster(hpd):
+    # m = 12 > 8 CTAs per cluster: CTAs take two rows each in turn; -inf rows
+    # land on a CTA's second row
+    rng = np.random.default_rng(12)
+    B, m, V = 7, 12, 1000
+    vals = rng.integers(-2, 3, size=(B, m, V)).astype(np.float32)
+    vals[1, 9, :] = -np.inf
+    vals[1, 9, :500] = np.nan
+    vals[2, 11, :] = np.nan
+    vals[3, 8, :] = -np.inf
+    logits = W.f32_to_bf16_bits(vals)
+    ref_tok0, _ = oracle.pmtp_accept(logits, np.zeros((B, m), np.int32))
+    drafts = W.mix_drafts(ref_tok0, V, 0.9, seed=13)
+    ref_tok, ref_acc = oracle.pmtp_accept(logits, drafts)
+    tok, acc = run_accept(hpd, logits, drafts)
+    np.testing.assert_array_equal(tok, ref_tok)
+    np.testing.assert_array_equal(acc, ref_acc)
+    assert ref_tok[1, 9] == 500 and ref_tok[3, 8] == 0
 
 
 def test_accept_misaligned_rows(hpd):
