@@ -497,45 +497,121 @@ def run_ours(args, world, rank, local):
                    "query_tokens_per_s": lay.B * lay.m / (lay_us * 1e-6),
                    "note": "attention call only, one L2-warm input replica"}
 
-    # ---- end to end: pinned host inputs in, results out, every step
-    host_q = torch.from_numpy(inp.q.view(np.int16)).pin_memory()
-    host_meta = [torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).pin_memory()
-                 for a in (inp.page_table, inp.branch_len, inp.prefix_cu, inp.branch_cu)]
-    host_logits = torch.from_numpy(logits_np.view(np.int16)).pin_memory()
-    host_drafts = torch.from_numpy(drafts_np).pin_memory()
-    host_out = torch.empty(op.out.shape, dtype=torch.bfloat16).pin_memory()
-    host_lse = torch.empty(op.lse.shape, dtype=torch.float32).pin_memory()
-    host_tok = torch.empty(out_tokens.shape, dtype=torch.int32).pin_memory()
-    host_acc = torch.empty(acc.shape, dtype=torch.int32).pin_memory()
+    # ---- end to end: pinned host inputs in, results out, every step.  Each
+    # step copies its inputs H2D in one packed copy (q, page table, lengths,
+    # offsets, logits, drafts), runs the attention and the acceptance through
+    # the C ABI, and copies its results D2H in one packed copy (out, lse,
+    # tokens, accepted lengths).  Two slots and three streams (H2D, compute,
+    # D2H) let a step's copies overlap the neighbouring steps' kernels; the
+    # resident prefix and paged KV rotate over the replicas as above.
+    def packed(sizes):
+        offs, o = [], 0
+        for n in sizes:
+            offs.append(o)
+            o += (n + 255) // 256 * 256
+        return offs, o
 
-    def h2d(r):
-        d = reps[r]
-        d.q.view(torch.int16).copy_(host_q, non_blocking=True)
-        for dst, src in zip((d.page_table, d.branch_len, d.prefix_cu, d.branch_cu), host_meta):
-            dst.copy_(src, non_blocking=True)
-        logits[r].view(torch.int16).copy_(host_logits, non_blocking=True)
-        drafts.copy_(host_drafts, non_blocking=True)
+    in_arrays = [np.ascontiguousarray(a) for a in (inp.q, inp.page_table.astype(np.int32),
+                                                    inp.branch_len.astype(np.int32),
+                                                    inp.prefix_cu.astype(np.int32),
+                                                    inp.branch_cu.astype(np.int32), logits_np,
+                                                    drafts_np.astype(np.int32))]
+    in_sizes = [a.nbytes for a in in_arrays]
+    in_offs, in_total = packed(in_sizes)
+    host_in = torch.zeros(in_total, dtype=torch.uint8).pin_memory()
+    for arr, o in zip(in_arrays, in_offs):
+        host_in[o:o + arr.nbytes].copy_(torch.from_numpy(arr.reshape(-1).view(np.uint8)))
+    rows = inp.B * inp.m
+    out_sizes = [rows * inp.H_q * inp.D * 2, rows * inp.H_q * 4, rows * 4, inp.B * 4]
+    out_offs, out_total = packed(out_sizes)
+    host_out = torch.empty(out_total, dtype=torch.uint8).pin_memory()
 
-    def d2h():
-        host_out.copy_(op.out, non_blocking=True)
-        host_lse.copy_(op.lse, non_blocking=True)
-        host_tok.copy_(out_tokens, non_blocking=True)
-        host_acc.copy_(acc, non_blocking=True)
+    def view(buf, off, n, dtype, shape):
+        return buf[off:off + n].view(dtype).view(shape)
 
-    h2d_bytes = sum(t.numel() * t.element_size()
-                    for t in [host_q, *host_meta, host_logits, host_drafts])
-    d2h_bytes = sum(t.numel() * t.element_size() for t in (host_out, host_lse, host_tok, host_acc))
-    def e2e_step(r, i):
-        h2d(r)
-        step(r)
-        d2h()
+    slots = []
+    for _ in range(2):
+        din = torch.empty(in_total, dtype=torch.uint8, device=dev)
+        dout = torch.empty(out_total, dtype=torch.uint8, device=dev)
+        i32 = torch.int32
+        slots.append(dict(
+            din=din, dout=dout,
+            q=view(din, in_offs[0], in_sizes[0], torch.bfloat16, (rows, inp.H_q, inp.D)),
+            pt=view(din, in_offs[1], in_sizes[1], i32, inp.page_table.shape),
+            bl=view(din, in_offs[2], in_sizes[2], i32, (inp.B,)),
+            pcu=view(din, in_offs[3], in_sizes[3], i32, (inp.n_docs + 1,)),
+            bcu=view(din, in_offs[4], in_sizes[4], i32, (inp.n_docs + 1,)),
+            lg=view(din, in_offs[5], in_sizes[5], torch.bfloat16, (inp.B, inp.m, VOCAB)),
+            dr=view(din, in_offs[6], in_sizes[6], i32, (inp.B, inp.m)),
+            out=view(dout, out_offs[0], out_sizes[0], torch.bfloat16, (rows, inp.H_q, inp.D)),
+            lse=view(dout, out_offs[1], out_sizes[1], torch.float32, (rows, inp.H_q)),
+            tok=view(dout, out_offs[2], out_sizes[2], i32, (inp.B, inp.m)),
+            acc=view(dout, out_offs[3], out_sizes[3], i32, (inp.B,))))
+    e2e_args = {}
 
-    ge_main = capture(S, 0, e2e_step)
-    ge_rem = capture(K % S, S, e2e_step) if K % S else None
+    def slot_args(s_i, r):
+        if (s_i, r) not in e2e_args:
+            sl, rep = slots[s_i], reps[r]
+            d = H.DeviceInputs(**{**rep.__dict__, "q": sl["q"], "page_table": sl["pt"],
+                                  "branch_len": sl["bl"], "prefix_cu": sl["pcu"],
+                                  "branch_cu": sl["bcu"]})
+            e2e_args[(s_i, r)] = (d, H.make_args(d, sl["out"], sl["lse"], op.workspace,
+                                                 op.workspace.numel()))
+        return e2e_args[(s_i, r)][1]
+
+    h2d_s = torch.cuda.Stream(device=dev)
+    d2h_s = torch.cuda.Stream(device=dev)
+
+    def e2e_capture(nsteps, offset):
+        g = torch.cuda.CUDAGraph()
+        events = []  # keep the events alive with the graph
+        with torch.cuda.graph(g, stream=stream):
+            h2d_s.wait_stream(stream)
+            d2h_s.wait_stream(stream)
+            comp, out_done = {}, {}
+            for i in range(nsteps):
+                s_i, r = i % 2, (offset + i) % R
+                sl = slots[s_i]
+                ev_in = torch.cuda.Event()
+                with torch.cuda.stream(h2d_s):
+                    if i >= 2:
+                        h2d_s.wait_event(comp[i - 2])   # the slot's inputs were consumed
+                    sl["din"].copy_(host_in, non_blocking=True)
+                    ev_in.record(h2d_s)
+                stream.wait_event(ev_in)
+                if i >= 2:
+                    stream.wait_event(out_done[i - 2])  # the slot's results were read out
+                H.hpd_branch_attn(slot_args(s_i, r), sh)
+                H.hpd_pmtp_accept(sl["lg"].data_ptr(), sl["dr"].data_ptr(), inp.B, inp.m, VOCAB,
+                                  sl["tok"].data_ptr(), sl["acc"].data_ptr(), sh)
+                comp[i] = torch.cuda.Event()
+                comp[i].record(stream)
+                with torch.cuda.stream(d2h_s):
+                    d2h_s.wait_event(comp[i])
+                    host_out.copy_(sl["dout"], non_blocking=True)
+                    out_done[i] = torch.cuda.Event()
+                    out_done[i].record(d2h_s)
+                events += [ev_in, comp[i], out_done[i]]
+            stream.wait_stream(h2d_s)
+            stream.wait_stream(d2h_s)
+        g._hpd_events = events
+        return g
+
+    h2d_bytes = sum(in_sizes)
+    d2h_bytes = sum(out_sizes)
+    ge_main = e2e_capture(S, 0)
+    ge_rem = e2e_capture(K % S, S) if K % S else None
+    with torch.cuda.stream(stream):
+        ge_main.replay()  # untimed first replay
+    torch.cuda.synchronize(dev)
     e2e_ms = timed(ge_main, ge_rem, n_main)
     err = op.errors(stream)
     if err:
         raise SystemExit(f"bench.py: device error flags {err:#x}")
+    # the results that came back are the library's (the last replayed step's slot)
+    last = slots[((K % S) - 1) % 2] if ge_rem is not None else slots[(S - 1) % 2]
+    if not torch.equal(host_out, last["dout"].cpu()):
+        raise SystemExit("bench.py: end-to-end results differ from the device copy")
 
     # ---- CPU baseline: the oracle on this host's cores (rank 0, N = 1 only)
     cpu = None
@@ -596,9 +672,11 @@ def run_ours(args, world, rank, local):
         },
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
                 "d2h_bytes_per_step": d2h_bytes,
-                "note": "q, page table, lengths, offsets, logits and drafts H2D from pinned "
-                        "host memory and out, lse, tokens, accepted lengths D2H every step; "
-                        "prefix KV and paged KV cache resident"},
+                "note": "every step: q, page table, lengths, offsets, logits and drafts H2D "
+                        "from pinned host memory in one packed copy, out, lse, tokens and "
+                        "accepted lengths D2H in one packed copy; two slots on H2D / compute "
+                        "/ D2H streams overlap a step's copies with the neighbouring steps' "
+                        "kernels; prefix KV and paged KV cache resident"},
         "gpu_launches": K * (n_launch + 1),
         "roofline": roof,
         "step_roofline": {"bytes": step_work["bytes"], "flops": step_work["flops"],
