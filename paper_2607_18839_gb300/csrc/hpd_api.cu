@@ -23,6 +23,7 @@ constexpr int kTargetCtas = kPlanSms * 4;  // warp-MMA prefix CTAs aimed for
 constexpr int kTcTileRows = 128;       // stacked rows of one tcgen05 prefix CTA
 constexpr int kMaxPrefixSplits = 8;
 constexpr int kLptWaves = 2;
+constexpr double kLptMinUs = 250.0;
 constexpr size_t kOrderSmemMax = 200 * 1024;
 constexpr int kSuffixSplitKeys = 1536;  // a suffix chunk holds at most ~this many keys
 constexpr int kMaxSuffixSplits = 8;
@@ -93,8 +94,12 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
     pl.S_p = best;
     // With at least kLptWaves units per SM, units of unequal length leave
     // SMs idle at the end; a one-CTA pass then orders them longest first
-    // (it holds the per-page and per-branch lengths in shared memory).
-    pl.lpt = ctas * best >= kLptWaves * kPlanSms &&
+    // (it holds the per-page and per-branch lengths in shared memory).  The
+    // pass costs about 10 us and saves a few percent of the kernel, so it
+    // runs only when the kernel is estimated at kLptMinUs or more.
+    const double est_us = static_cast<double>(ctas) * best * (ceil_div(nb, best) + 1) *
+                          block_us / kPlanSms;
+    pl.lpt = ctas * best >= kLptWaves * kPlanSms && est_us >= kLptMinUs &&
              hpd::unit_order_smem_bytes(a->n_docs, a->B, pl.tiles_max) <= kOrderSmemMax;
   } else {
     const long long stacked = static_cast<long long>(a->B) * a->m * pl.G;

@@ -5,6 +5,7 @@ import ctypes
 import os
 import re
 
+import numpy as np
 import pytest
 
 from paper_2607_18839_gb300 import build as B
@@ -132,13 +133,22 @@ def _workload_args(inp):
     return a
 
 
+def big_workload():
+    """Three times the 32-page preset's pages (96 pages, 24 branches each)."""
+    from paper_2607_18839_gb300 import workloads as W
+    rng = np.random.default_rng(77)
+    P = rng.integers(1024, 3073, size=96)
+    s = np.clip(np.round(rng.lognormal(4.5, 0.8, size=96 * 24)), 1, 1024).astype(np.int64)
+    return W.build_inputs(P, [24] * 96, s, 8, 16, 2, 128, seed=78, max_pages=65, name="c4x3")
+
+
 def test_launch_plan_of_the_workloads(lib):
     # host-only planning: which kernels one call launches (no GPU needed)
     from paper_2607_18839_gb300 import workloads as W
     expect = {
         "c1": ["branch_attn_tc"],                        # one wave, no key split
         "c2": ["branch_attn_tc", "merge_splits"],        # few tiles: keys split, then merged
-        "c4": ["unit_order", "branch_attn_tc"],          # >= 2 units per SM: longest first
+        "c4": ["branch_attn_tc"],                        # the order pass would not pay
         "c5": ["branch_attn_tc"],
     }
     for name, kernels in expect.items():
@@ -147,6 +157,9 @@ def test_launch_plan_of_the_workloads(lib):
         got = [hpd.hpd_branch_attn_kernel_name(a, k) for k in range(n)]
         assert got == kernels, (name, got)
         assert hpd.hpd_branch_attn_kernel_name(a, n) is None
+    # a large step (96 pages) orders its work units longest first
+    assert [hpd.hpd_branch_attn_kernel_name(_workload_args(big_workload()), k) for k in range(2)] == [
+        "unit_order", "branch_attn_tc"]
     # head ratios that do not divide 128 take the warp-MMA stages
     g3 = W.build_inputs([200], [3], [4, 0, 33], 3, 6, 2, 128, seed=1)
     a = _workload_args(g3)

@@ -201,6 +201,24 @@ def test_paged_prefix_bad_page_id_is_flagged(hpd):
     assert np.all(np.isfinite(out))
 
 
+def test_parity_large_step_with_ordered_units(hpd):
+    # 96 pages: long enough that the work units are ordered longest first
+    from test_abi import big_workload
+    inp = big_workload()
+    d = hpd.DeviceInputs.from_host(inp)
+    op = hpd.BranchAttn(d)
+    names = [hpd.hpd_branch_attn_kernel_name(op.args, k)
+             for k in range(hpd.hpd_branch_attn_launches(op.args))]
+    assert names == ["unit_order", "branch_attn_tc"]
+    out, lse = op()
+    torch.cuda.synchronize()
+    assert op.errors() == 0
+    sel = np.array(sample_branches(inp, k=10), dtype=np.int32)
+    ref_out, ref_lse = oracle.branch_attn(inp, branch_sel=sel)
+    compare(inp, out.float().cpu().numpy(), lse.cpu().numpy(), ref_out, ref_lse,
+            rows=branch_rows(inp, sel))
+
+
 def test_c3_full_oracle_elementwise(hpd):
     inp = W.make_config("c3")
     ref_out, ref_lse = oracle.branch_attn(inp)
