@@ -18,15 +18,19 @@ import oracle  # noqa: E402
 from paper_2607_18839_gb300 import workloads as W  # noqa: E402
 
 
-def main():
-    inp = W.make_config("c1")
+def layout_case():
+    """Two pages with their layout branches and content branches, the prefix
+    paged and shared with the layout branches (paged prefix, fork limits)."""
+    return W.build_layout_inputs([37, 64], [20, 0], [2, 1], [5, 17, 3], 3, 4, 2, 64, seed=3)
+
+
+def write(inp, path, header):
     out, lse = oracle.branch_attn(inp)
-    path = os.path.join(HERE, "c1_oracle.txt")
     with open(path, "w") as f:
-        f.write("# fp64 oracle on workload c1 (seed 1001): one page, prefix 256, 4 branches\n")
-        f.write("# with private histories 8/16/24/32, m=1, H_q=8, H_kv=2, D=64.\n")
+        for line in header:
+            f.write(f"# {line}\n")
         f.write("# Written by tests/golden/make_golden.py from oracle/ only.\n")
-        f.write("# lines: 'lse row head value' and 'out row head c value' (heads 0 and 7)\n")
+        f.write(f"# lines: 'lse row head value' and 'out row head c value' (heads 0 and {inp.H_q - 1})\n")
         for r in range(inp.rows):
             for h in range(inp.H_q):
                 f.write(f"lse {r} {h} {lse[r, h]:.17g}\n")
@@ -35,6 +39,16 @@ def main():
                 for c in range(inp.D):
                     f.write(f"out {r} {h} {c} {out[r, h, c]:.17g}\n")
     print("wrote", path)
+
+
+def main():
+    write(W.make_config("c1"), os.path.join(HERE, "c1_oracle.txt"),
+          ["fp64 oracle on workload c1 (seed 1001): one page, prefix 256, 4 branches",
+           "with private histories 8/16/24/32, m=1, H_q=8, H_kv=2, D=64."])
+    write(layout_case(), os.path.join(HERE, "layout_oracle.txt"),
+          ["fp64 oracle on a small layout-branch workload (seed 3): pages with vision 37 / 64",
+           "and layout 20 / 0 tokens, 2 / 1 content branches, m=3, H_q=4, H_kv=2, D=64; the",
+           "prefix is paged and shared with each page's layout branch."])
 
 
 if __name__ == "__main__":
