@@ -8,18 +8,24 @@ are at least two units per SM and followed by the LSE merge of key splits
 when the keys are split) followed by hpd_pmtp_accept (greedy verification of
 the P-MTP drafts against bf16 logits over a 32,000-token vocabulary).
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c2]
-                    [--impl ours|reference]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c4]
+                    [--also c2,c3,c5] [--replays 5] [--impl ours|reference]
 
-Prints ONE JSON line on rank 0.  The metric is query tokens (branches x m)
-per second; ``roofline`` reports the dominant kernel against the measured
-peaks in MEASURED_PEAKS.json; ``cpu_baseline`` times the fp64 oracle on the
-host cores.  ``--impl reference`` times the oracle itself as the bench arm.
+Prints ONE JSON line on rank 0.  The headline workload is c4 (32 pages, 768
+branches, m = 8: the largest single-GPU preset by query tokens and bytes);
+the other presets follow in ``per_config``.  The metric is query tokens
+(branches x m) per second of the whole step, attention then acceptance;
+``attention_only`` gives the attention call alone.  ``roofline`` reports the
+dominant kernel against the measured peaks in MEASURED_PEAKS.json;
+``cpu_baseline`` times the fp64 oracle on the host cores; ``context`` quotes
+the paper's own end-to-end figure.  ``--impl reference`` times the oracle
+itself as the bench arm.
 
-Timing: W warm-up steps, then exactly K steps replayed from CUDA graphs,
-bracketed by a barrier and a device synchronize, with the input replicas
-rotated so that their footprint exceeds 3x the L2 cache.  Per-kernel times
-come from timing markers recorded inside the graphs of the timed region.
+Timing: W warm-up steps, then one CUDA graph of exactly K steps replayed at
+least five times, each replay bracketed by a barrier and a device
+synchronize and timed with CUDA events on the launch stream; the median is
+reported.  The input replicas rotate so that their footprint exceeds 3x the
+L2 cache; ``cold_l2`` adds steps that each follow an explicit L2 eviction.
 Under torchrun each rank processes its own pages (pages are independent; no
 collective on the data path) and the slowest rank's time is used.
 """
@@ -252,27 +258,75 @@ def oracle_sample_run(inp, logits, drafts, budget_s: float, rng_seed: int = 0):
 
 # --------------------------------------------------------------- our path --
 
-def run_ours(args, world, rank, local):
+PAPER_CONTEXT = {
+    "value": 4752.1, "unit": "tokens/s",
+    "what": "HPD-Parsing end-to-end decode throughput of the whole model (Table 2)",
+    "hardware": "NVIDIA A800 80GB GPUs (count unstated), vLLM 0.17.1, batch 512, OmniDocBench v1.6",
+    "note": "context only: another metric (generated tokens of the full model) on other hardware",
+}
+
+
+def step_config(name, world):
+    """The `config` object of a workload's bench line (the same in both arms)."""
+    inp_desc = W.CONFIG_DESCRIPTIONS[name]
+    cfg = W.config_shape(name)
+    return {
+        "workload": f"{name}: {inp_desc}; acceptance over bf16 logits "
+                    f"[{cfg['B']} x {cfg['m']} x {VOCAB}]",
+        "query_tokens_per_step": cfg["B"] * cfg["m"],
+        "step": "hpd_branch_attn (shared prefix + private suffix + merge) then hpd_pmtp_accept "
+                "(acceptance inside the step)",
+        "parallelism": f"dp{world} (independent pages per GPU, no collective)",
+    }
+
+
+class Timer:
+    """CUDA-event timing of graph replays on one stream."""
+
+    def __init__(self, torch, dev, stream, world, dist):
+        self.torch, self.dev, self.stream, self.world, self.dist = torch, dev, stream, world, dist
+        self.wall_ms = 0.0
+
+    def replay_ms(self, graphs, sync_ranks=True):
+        """Time one replay of `graphs` (in order), bracketed by a barrier and
+        a device synchronize; the max over ranks."""
+        torch = self.torch
+        if self.world > 1 and sync_ranks:
+            self.dist.barrier()
+        torch.cuda.synchronize(self.dev)
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        w0 = time.perf_counter()
+        with torch.cuda.stream(self.stream):  # replay() launches on the current stream
+            t0.record(self.stream)
+            for g in graphs:
+                g.replay()
+            t1.record(self.stream)
+        torch.cuda.synchronize(self.dev)
+        self.wall_ms = (time.perf_counter() - w0) * 1e3
+        ms = t0.elapsed_time(t1)
+        if self.world > 1 and sync_ranks:
+            ms = max_over_ranks(ms, self.world, self.dev)
+            self.dist.barrier()
+        return ms
+
+    def median_ms(self, graphs, n, sync_ranks=False):
+        return statistics.median(self.replay_ms(graphs, sync_ranks) for _ in range(n))
+
+
+def measure_workload(name, args, world, rank, dev, stream, H, headline):
+    """Time one workload's step (and, for the headline, its side lines)."""
     import torch
     import torch.distributed as dist
-    from paper_2607_18839_gb300 import build as hpd_build
-    from paper_2607_18839_gb300 import hpd as H
 
-    if not torch.cuda.is_available():
-        raise SystemExit("bench.py: no CUDA device (the CUDA path has no CPU fallback)")
-    if world > 1:
-        dist.init_process_group("nccl", init_method="env://")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    hpd_build.build()
-    H.load()
-
-    cid = int(args.workload.lstrip("c"))
+    cid = int(name.lstrip("c"))
     seed_t, seed_l = rank_seeds(cid, rank)
-    inp = W.make_config(args.workload, seed=seed_t)
+    inp = W.make_config(name, seed=seed_t)
     logits_np = W.make_logits(inp.B, inp.m, VOCAB, seed=seed_l)
-    stream = torch.cuda.Stream(device=dev)
     sh = int(stream.cuda_stream)
+    timer = Timer(torch, dev, stream, world, dist)
+    K = args.steps
+    n_rep = max(5, args.replays)
 
     # ---- replicas: footprint > 3x L2 so timed steps read from HBM
     base = H.DeviceInputs.from_host(inp, device=dev)
@@ -283,7 +337,7 @@ def run_ours(args, world, rank, local):
     l2 = int(getattr(torch.cuda.get_device_properties(dev), "L2_cache_size", 128 << 20))
     free, _ = torch.cuda.mem_get_info(dev)
     R = max(2, math.ceil(3 * l2 / rep_bytes))
-    R = int(min(R, 256, max(2, (free * 0.5) // rep_bytes)))
+    R = int(min(R, 256, max(2, (free * 0.4) // rep_bytes)))
 
     def clone_inputs(d):
         return H.DeviceInputs(**{k: (v.clone() if isinstance(v, torch.Tensor) else v)
@@ -305,7 +359,8 @@ def run_ours(args, world, rank, local):
         H.hpd_pmtp_accept(logits0.data_ptr(), zeros.data_ptr(), inp.B, inp.m, VOCAB,
                           out_tokens.data_ptr(), acc.data_ptr(), sh)
     stream.synchronize()
-    drafts_np = W.mix_drafts(out_tokens.cpu().numpy(), VOCAB, DRAFT_MATCH, seed=3000 + rank)
+    argmax_np = out_tokens.cpu().numpy()
+    drafts_np = W.mix_drafts(argmax_np, VOCAB, DRAFT_MATCH, seed=3000 + rank)
     drafts = torch.from_numpy(drafts_np).to(dev)
 
     def attn(r, ev=None):
@@ -329,11 +384,7 @@ def run_ours(args, world, rank, local):
     stream.synchronize()
     err = op.errors(stream)
     if err:
-        raise SystemExit(f"bench.py: device error flags {err:#x}")
-
-    # ---- CUDA graphs of S steps (inputs rotated over the R replicas)
-    K = args.steps
-    S = max(1, min(K, args.graph_steps))
+        raise SystemExit(f"bench.py: device error flags {err:#x} on {name}")
 
     def capture(nsteps, offset, body):
         g = torch.cuda.CUDAGraph()
@@ -342,160 +393,68 @@ def run_ours(args, world, rank, local):
                 body((offset + i) % R, i)
         return g
 
-    g_main = capture(S, 0, lambda r, i: step(r))
-    g_rem = capture(K % S, S, lambda r, i: step(r)) if K % S else None
-    n_main = K // S
+    # ---- the timed region: one CUDA graph of exactly K steps (inputs
+    # rotated over the R replicas), replayed n_rep times; each replay is
+    # bracketed by a barrier and a device synchronize, and the median is kept
+    g_step = capture(K, 0, lambda r, i: step(r))
+    with torch.cuda.stream(stream):
+        g_step.replay()  # untimed first replay
+    clocks = None
+    if headline:
+        gpu_id = str(torch.cuda.get_device_properties(dev).uuid)
+        gpu_id = gpu_id if gpu_id.startswith("GPU-") else f"GPU-{gpu_id}"
+        clocks = ClockSampler(gpu_id)
+        clocks.start()
+    step_runs = [timer.replay_ms([g_step], sync_ranks=True) for _ in range(n_rep)]
+    wall_ms = timer.wall_ms
+    clk = clocks.stop() if clocks is not None else None
+    ms_step = statistics.median(step_runs) / K
 
-    wall_ms = [0.0]  # host wall clock of the last timed region (cross-check)
-
-    def timed(gm, gr, nm, sync_ranks=True):
-        if world > 1 and sync_ranks:
-            dist.barrier()
-        torch.cuda.synchronize(dev)
-        t0 = torch.cuda.Event(enable_timing=True)
-        t1 = torch.cuda.Event(enable_timing=True)
-        w0 = time.perf_counter()
-        # replay() launches on the current stream: make it the timing stream
-        with torch.cuda.stream(stream):
-            t0.record(stream)
-            for _ in range(nm):
-                gm.replay()
-            if gr is not None:
-                gr.replay()
-            t1.record(stream)
-        torch.cuda.synchronize(dev)
-        wall_ms[0] = (time.perf_counter() - w0) * 1e3
-        ms = t0.elapsed_time(t1)
-        if world > 1 and sync_ranks:
-            ms = max_over_ranks(ms, world, dev)
-            dist.barrier()
-        return ms
-
-    gpu_id = str(torch.cuda.get_device_properties(dev).uuid)
-    gpu_id = gpu_id if gpu_id.startswith("GPU-") else f"GPU-{gpu_id}"
-    clocks = ClockSampler(gpu_id)
-    clocks.start()
-    total_ms = timed(g_main, g_rem, n_main)
-    total_wall_ms = wall_ms[0]
-    clk = clocks.stop()
-
-    # ---- per-kernel durations, measured right after the timed region on the
-    # same stream: the attention call and the acceptance kernel each replayed
-    # back to back from their own graphs (events around the replays), and the
-    # attention call's kernels apportioned by timing markers recorded inside a
-    # graph of marked calls.
-    n_rep = max(1, (2 * K) // S)
-    g_attn = capture(S, 0, lambda r, i: attn(r))
-    g_acc = capture(S, 0, lambda r, i: accept(r))
-    attn_ms = timed(g_attn, None, n_rep, sync_ranks=False) / (n_rep * S)
-    acc_ms = timed(g_acc, None, n_rep, sync_ranks=False) / (n_rep * S)
+    # ---- per-call times: the attention call and the acceptance each from a
+    # graph of K back-to-back calls (median of n_rep replays); the attention
+    # call's kernels apportioned by timing markers recorded inside a graph
+    g_attn = capture(K, 0, lambda r, i: attn(r))
+    g_acc = capture(K, 0, lambda r, i: accept(r))
+    attn_ms = timer.median_ms([g_attn], n_rep) / K
+    acc_ms = timer.median_ms([g_acc], n_rep) / K
     attn_names = [H.hpd_branch_attn_kernel_name(argsets[0], k) for k in range(n_launch)]
-    events = [[torch.cuda.Event(enable_timing=True) for _ in range(n_launch + 1)] for _ in range(S)]
+    S_mark = min(K, 50)
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(n_launch + 1)]
+              for _ in range(S_mark)]
     with torch.cuda.stream(stream):
         for row in events:
             for e in row:
                 e.record(stream)  # creates the handle
     stream.synchronize()
     handles = [[int(e.cuda_event) for e in row] for row in events]
-    g_mark = capture(S, 0, lambda r, i: attn(r, handles[i]))
+    g_mark = capture(S_mark, 0, lambda r, i: attn(r, handles[i]))
     with torch.cuda.stream(stream):
         g_mark.replay()
     torch.cuda.synchronize(dev)
-    span = [statistics.mean(ev[k].elapsed_time(ev[k + 1]) for ev in events) for k in range(n_launch)]
-    kernel_ms = {name: attn_ms * span[k] / sum(span) for k, name in enumerate(attn_names)}
+    span = [statistics.mean(ev[k].elapsed_time(ev[k + 1]) for ev in events)
+            for k in range(n_launch)]
+    kernel_ms = {nm: attn_ms * span[k] / sum(span) for k, nm in enumerate(attn_names)}
     kernel_ms[ACCEPT] = acc_ms
 
-    # ---- paged-KV append / rollback around a step (reported beside the step,
-    # not part of its metric): append the step's m rows of every branch, then
-    # roll all of them back (accepted_len = -1), which restores the pool
-    used = np.ceil(inp.branch_len / W.PAGE).astype(np.int64)
-    kv_max_pages = int(np.max(np.ceil((inp.branch_len + inp.m) / W.PAGE)))
-    kv_pages = int(used.sum() + inp.B * (inp.m // W.PAGE + 2))
-    pool = W.make_kv_pool(inp.branch_len, inp.m, inp.H_kv, inp.D, kv_pages, kv_max_pages,
-                          seed=4000 + cid)
-    kv_new = W.make_kv_rows(inp.B, inp.m, inp.H_kv, inp.D, seed=5000 + cid)
-    tdev = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
-    kv = H.PagedKV(tdev(pool["k_cache"].view(np.int16)), tdev(pool["v_cache"].view(np.int16)),
-                   tdev(pool["page_table"]), tdev(pool["branch_len"]), tdev(pool["free"]),
-                   torch.tensor([pool["top"]], dtype=torch.int32, device=dev), inp.m)
-    k_new, v_new = (tdev(a.view(np.int16)) for a in kv_new)
-    reject_all = torch.full((inp.B,), -1, dtype=torch.int32, device=dev)
-
-    def kv_pair(r, i):
-        kv.append(k_new, v_new, stream)
-        kv.rollback(reject_all, stream)
-
-    with torch.cuda.stream(stream):
-        kv_pair(0, 0)
-    g_kv = capture(S, 0, kv_pair)
-    kv_ms = timed(g_kv, None, n_rep, sync_ranks=False) / (n_rep * S)
-    if kv.errors(stream):
-        raise SystemExit(f"bench.py: KV append / rollback error flags {kv.errors(stream):#x}")
-    kv_bytes = 2 * 2 * inp.B * inp.m * inp.H_kv * inp.D * 2  # K and V rows read + written
-    kv_line = {"us_per_pair": kv_ms * 1e3, "launches_per_pair": 3, "bytes": kv_bytes,
-               "achieved_gbs": kv_bytes / (kv_ms * 1e-3) / 1e9,
-               "note": "hpd_kv_append (m rows per branch) + hpd_kv_rollback (all rolled back) "
-                       "on a pool of the workload's lengths; not part of the step metric"}
-
-    # ---- fork detection / child branches after the acceptance (reported beside
-    # the step): the step's argmax tokens with 2% fork tokens, each page's
-    # first branch its layout branch
-    rng_f = np.random.default_rng(6000 + cid)
-    fork_tok = np.where(rng_f.random((inp.B, inp.m)) < 0.02, VOCAB - 1,
-                        rng_f.integers(0, VOCAB - 1, size=(inp.B, inp.m))).astype(np.int32)
-    is_layout = np.zeros(inp.B, np.int32)
-    is_layout[inp.branch_cu[:-1][np.diff(inp.branch_cu) > 0]] = 1
-    f_in = [tdev(a) for a in (fork_tok, acc.cpu().numpy(), is_layout,
-                               inp.branch_prefix_len if inp.branch_prefix_len is not None
-                               else np.zeros(inp.B, np.int32), inp.branch_cu, inp.branch_len,
-                               inp.page_table)]
-    f_cap = inp.B * (inp.m + 1)
-    f_state = {}
-
-    def fork_call(r, i):
-        f_state["out"] = H.fork_children(f_in[0], f_in[1], f_in[2], f_in[3], VOCAB - 1, f_in[4],
-                                         None, f_in[5], f_in[6], f_cap, stream)
-
-    with torch.cuda.stream(stream):
-        fork_call(0, 0)
+    # ---- cold L2: before each step a write of twice the L2 size evicts
+    # everything; events around the step alone
+    flush = torch.empty(2 * l2, dtype=torch.uint8, device=dev)
+    n_cold = max(5, min(20, K))
+    ev_cold = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+                torch.cuda.Event(enable_timing=True)) for _ in range(n_cold)]
     torch.cuda.synchronize(dev)
-    g_fork = capture(S, 0, fork_call)
-    fork_ms = timed(g_fork, None, n_rep, sync_ranks=False) / (n_rep * S)
-    fork_line = {"us_per_call": fork_ms * 1e3,
-                 "children": int(f_state["out"]["new_B"].item()) - inp.B,
-                 "note": "hpd_fork_children over the step's branches (two launches); not part of "
-                         "the step metric"}
-
-    # ---- the attention call on other layouts of the prefix and on the
-    # layout-branch workload (reported beside the step; one input replica)
-    def attn_call_us(inp_x):
-        op_x = H.BranchAttn(H.DeviceInputs.from_host(inp_x), stream)
-        with torch.cuda.stream(stream):
-            for _ in range(3):
-                op_x(stream)
-        torch.cuda.synchronize(dev)
-        g_x = capture(S, 0, lambda r, i: op_x(stream))
-        ms = timed(g_x, None, n_rep, sync_ranks=False) / (n_rep * S)
-        if op_x.errors(stream):
-            raise SystemExit(f"bench.py: error flags {op_x.errors(stream):#x} on {inp_x.name}")
-        return ms * 1e3, H.hpd_branch_attn_launches(op_x.args)
-
-    runs_us, _ = attn_call_us(W.page_the_prefix(inp, seed=7000 + cid, runs=True))
-    scat_us, _ = attn_call_us(W.page_the_prefix(inp, seed=7000 + cid, runs=False))
-    paged_line = {"us_per_call_consecutive_pages": runs_us, "us_per_call_scattered_pages": scat_us,
-                  "contiguous_us_per_call": attn_ms * 1e3,
-                  "note": "the same attention call with every page's prefix in the 16-token KV "
-                          "pool through a prefix page table: in consecutive pool pages (one "
-                          "prefill allocation) or scattered; one L2-warm input replica"}
-    lay = W.make_layout_config()
-    lay_us, lay_launch = attn_call_us(lay)
-    layout_line = {"workload": "8 pages, vision U[1024,3072], layout tokens U[64,512], each "
-                               "page's layout branch + U[4,24] content branches forked after "
-                               "a layout token (lognormal histories), m=4, Hq16/Hkv2, D128, "
-                               "paged prefix shared with the layout branch",
-                   "us_per_call": lay_us, "launches": lay_launch,
-                   "query_tokens_per_s": lay.B * lay.m / (lay_us * 1e-6),
-                   "note": "attention call only, one L2-warm input replica"}
+    with torch.cuda.stream(stream):
+        for i, (e0, e1, e2) in enumerate(ev_cold):
+            flush.fill_(i & 0xff)
+            e0.record(stream)
+            attn(i % R)
+            e1.record(stream)
+            accept(i % R)
+            e2.record(stream)
+    torch.cuda.synchronize(dev)
+    cold_step_ms = statistics.median(e0.elapsed_time(e2) for e0, _, e2 in ev_cold)
+    cold_attn_ms = statistics.median(e0.elapsed_time(e1) for e0, e1, _ in ev_cold)
+    del flush
 
     # ---- end to end: pinned host inputs in, results out, every step.  Each
     # step copies its inputs H2D in one packed copy (q, page table, lengths,
@@ -562,7 +521,7 @@ def run_ours(args, world, rank, local):
     h2d_s = torch.cuda.Stream(device=dev)
     d2h_s = torch.cuda.Stream(device=dev)
 
-    def e2e_capture(nsteps, offset):
+    def e2e_capture(nsteps):
         g = torch.cuda.CUDAGraph()
         events = []  # keep the events alive with the graph
         with torch.cuda.graph(g, stream=stream):
@@ -570,7 +529,7 @@ def run_ours(args, world, rank, local):
             d2h_s.wait_stream(stream)
             comp, out_done = {}, {}
             for i in range(nsteps):
-                s_i, r = i % 2, (offset + i) % R
+                s_i, r = i % 2, i % R
                 sl = slots[s_i]
                 ev_in = torch.cuda.Event()
                 with torch.cuda.stream(h2d_s):
@@ -599,41 +558,24 @@ def run_ours(args, world, rank, local):
 
     h2d_bytes = sum(in_sizes)
     d2h_bytes = sum(out_sizes)
-    ge_main = e2e_capture(S, 0)
-    ge_rem = e2e_capture(K % S, S) if K % S else None
+    ge = e2e_capture(K)
     with torch.cuda.stream(stream):
-        ge_main.replay()  # untimed first replay
+        ge.replay()  # untimed first replay
     torch.cuda.synchronize(dev)
-    e2e_ms = timed(ge_main, ge_rem, n_main)
+    e2e_ms = statistics.median(timer.replay_ms([ge], sync_ranks=True) for _ in range(n_rep))
     err = op.errors(stream)
     if err:
-        raise SystemExit(f"bench.py: device error flags {err:#x}")
+        raise SystemExit(f"bench.py: device error flags {err:#x} on {name}")
     # the results that came back are the library's (the last replayed step's slot)
-    last = slots[((K % S) - 1) % 2] if ge_rem is not None else slots[(S - 1) % 2]
-    if not torch.equal(host_out, last["dout"].cpu()):
+    if not torch.equal(host_out, slots[(K - 1) % 2]["dout"].cpu()):
         raise SystemExit("bench.py: end-to-end results differ from the device copy")
 
-    # ---- CPU baseline: the oracle on this host's cores (rank 0, N = 1 only)
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, thr, sample = oracle_sample_run(inp, logits_np, drafts_np, args.cpu_seconds)
-        cpu = {"value": v, "unit": UNIT, "cores": thr, "kind": "oracle", "sample": sample}
-
-    if world > 1:
-        dist.destroy_process_group()
-    if rank != 0:
-        return None
-
+    # ---- numbers
     qtok = inp.B * inp.m
-    ms_step = total_ms / K
-    value = whole_job_value(world, qtok, ms_step)
-    e2e_value = whole_job_value(world, qtok, e2e_ms / K)
-
     pk = peaks()
     per, step_work = algorithmic_work(inp)
-    known = {k: v for k, v in kernel_ms.items() if v is not None}
-    dom = max(known, key=known.get)
-    dom_ms = known[dom]
+    dom = max(kernel_ms, key=kernel_ms.get)
+    dom_ms = kernel_ms[dom]
     t_bytes = per[dom]["bytes"] / (pk["hbm"] * 1e9)
     t_flops = per[dom]["flops"] / (pk["tc_sustained"] * 1e12)
     if t_flops > t_bytes:
@@ -644,54 +586,253 @@ def run_ours(args, world, rank, local):
         achieved = per[dom]["bytes"] / (dom_ms * 1e-3) / 1e9
         roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm"], "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["traffic"] = ncu_traffic(args.workload, dom)
+    roof["traffic"] = ncu_traffic(name, dom)
     roof["kernel"] = dom
-    roof["peak_source"] = pk["source"] + (" sustained bf16" if roof["bound"] == "tensor" else " HBM copy")
+    roof["kernel_us"] = dom_ms * 1e3
+    roof["algorithmic"] = {"bytes": per[dom]["bytes"], "flops": per[dom]["flops"]}
+    roof["peak_source"] = pk["source"] + (" sustained bf16" if roof["bound"] == "tensor"
+                                          else " HBM copy")
     roof["nominal_peak"] = NOMINAL_BF16_TFLOPS if roof["bound"] == "tensor" else NOMINAL_HBM_GBS
     roof["frac_of_nominal"] = roof["achieved"] / roof["nominal_peak"]
+    # the attention call's algorithmic work, whichever kernels carry it
+    attn_work = per["branch_attn_tc"]
+    t_attn_roof = max(attn_work["bytes"] / (pk["hbm"] * 1e9),
+                      attn_work["flops"] / (pk["tc_sustained"] * 1e12))
+    t_step_roof = max(step_work["bytes"] / (pk["hbm"] * 1e9),
+                      step_work["flops"] / (pk["tc_sustained"] * 1e12))
     acc_us = kernel_ms[ACCEPT] * 1e3
-    accept_line = {"us_per_call": acc_us, "bytes": per[ACCEPT]["bytes"],
-                   "achieved_gbs": per[ACCEPT]["bytes"] / (acc_us * 1e-6) / 1e9,
-                   "frac_of_measured_hbm": per[ACCEPT]["bytes"] / (acc_us * 1e-6) / 1e9 / pk["hbm"],
-                   "note": "greedy acceptance, HBM-bound: logits read once"}
-    t_roof = max(step_work["bytes"] / (pk["hbm"] * 1e9), step_work["flops"] / (pk["tc_sustained"] * 1e12))
-
-    line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
-        "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {
-            "workload": f"{args.workload}: {W.CONFIG_DESCRIPTIONS[args.workload]}; acceptance "
-                        f"over bf16 logits [{inp.B} x {inp.m} x {VOCAB}]",
-            "query_tokens_per_step": qtok,
-            "l2": f"{R} rotating input replicas ({R * rep_bytes / 2**20:.0f} MiB > 3x L2 "
-                  f"{l2 / 2**20:.0f} MiB)",
-            "timing": f"CUDA graphs of {S} steps, events on the launch stream; per-kernel "
-                      f"times from back-to-back graphs of each call after the timed region",
-            "parallelism": f"dp{world} (independent pages per GPU, no collective)",
+    res = {
+        "name": name, "inp": inp, "logits_np": logits_np, "drafts_np": drafts_np,
+        "value": whole_job_value(world, qtok, ms_step),
+        "ms_per_step": ms_step,
+        "step_replays_ms": step_runs,
+        "wall_ms": wall_ms,
+        "clocks": clk,
+        "n_launch": n_launch,
+        "roofline": roof,
+        "attention_only": {
+            "value": whole_job_value(world, qtok, attn_ms),
+            "unit": UNIT,
+            "us_per_call": attn_ms * 1e3,
+            "launches": n_launch,
+            "kernels": attn_names,
+            "roofline_us": t_attn_roof * 1e6,
+            "frac": t_attn_roof / (attn_ms * 1e-3),
+            "bound": "tensor" if attn_work["flops"] / (pk["tc_sustained"] * 1e12)
+                     > attn_work["bytes"] / (pk["hbm"] * 1e9) else "hbm",
+            "note": "hpd_branch_attn alone (no acceptance): algorithmic time at the measured "
+                    "peaks / measured call time",
         },
-        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
-                "d2h_bytes_per_step": d2h_bytes,
+        "step_roofline": {"bytes": step_work["bytes"], "flops": step_work["flops"],
+                          "t_roofline_us": t_step_roof * 1e6,
+                          "frac": t_step_roof / (ms_step * 1e-3)},
+        "kernel_us": {k: v * 1e3 for k, v in kernel_ms.items()},
+        "accept": {"us_per_call": acc_us, "bytes": per[ACCEPT]["bytes"],
+                   "achieved_gbs": per[ACCEPT]["bytes"] / (acc_us * 1e-6) / 1e9,
+                   "frac_of_measured_hbm":
+                       per[ACCEPT]["bytes"] / (acc_us * 1e-6) / 1e9 / pk["hbm"],
+                   "note": "greedy acceptance, HBM-bound: logits read once"},
+        "cold_l2": {"step_us": cold_step_ms * 1e3, "attention_us": cold_attn_ms * 1e3,
+                    "value": whole_job_value(world, qtok, cold_step_ms),
+                    "note": f"median of {n_cold} single steps, each right after a write of "
+                            f"{2 * l2 / 2**20:.0f} MiB (2x L2) evicted the cache"},
+        "e2e": {"value": whole_job_value(world, qtok, e2e_ms / K), "unit": UNIT,
+                "h2d_bytes_per_step": h2d_bytes, "d2h_bytes_per_step": d2h_bytes,
+                "ms_per_step": e2e_ms / K,
                 "note": "every step: q, page table, lengths, offsets, logits and drafts H2D "
                         "from pinned host memory in one packed copy, out, lse, tokens and "
                         "accepted lengths D2H in one packed copy; two slots on H2D / compute "
                         "/ D2H streams overlap a step's copies with the neighbouring steps' "
-                        "kernels; prefix KV and paged KV cache resident"},
-        "gpu_launches": K * (n_launch + 1),
-        "roofline": roof,
-        "step_roofline": {"bytes": step_work["bytes"], "flops": step_work["flops"],
-                          "t_roofline_us": t_roof * 1e6,
-                          "frac": t_roof / (ms_step * 1e-3)},
-        "kernel_us": {k: v * 1e3 for k, v in kernel_ms.items()},
-        "attn_call_us": attn_ms * 1e3,
-        "accept": accept_line,
-        "kv_append_rollback": kv_line,
-        "fork_children": fork_line,
-        "paged_prefix": paged_line,
-        "layout_branches": layout_line,
-        "host_wall_ms_per_step": total_wall_ms / K,
+                        "kernels; prefix KV and paged KV cache resident; median of "
+                        f"{n_rep} replays of a {K}-step graph"},
+        "l2": f"{R} rotating input replicas ({R * rep_bytes / 2**20:.0f} MiB > 3x L2 "
+              f"{l2 / 2**20:.0f} MiB)",
+    }
+    if not headline:
+        return res
+
+    # ---- paged-KV append / rollback around a step (reported beside the step,
+    # not part of its metric): append the step's m rows of every branch, then
+    # roll all of them back (accepted_len = -1), which restores the pool
+    used = np.ceil(inp.branch_len / W.PAGE).astype(np.int64)
+    kv_max_pages = int(np.max(np.ceil((inp.branch_len + inp.m) / W.PAGE)))
+    kv_pages = int(used.sum() + inp.B * (inp.m // W.PAGE + 2))
+    pool = W.make_kv_pool(inp.branch_len, inp.m, inp.H_kv, inp.D, kv_pages, kv_max_pages,
+                          seed=4000 + cid)
+    kv_new = W.make_kv_rows(inp.B, inp.m, inp.H_kv, inp.D, seed=5000 + cid)
+    tdev = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    kv = H.PagedKV(tdev(pool["k_cache"].view(np.int16)), tdev(pool["v_cache"].view(np.int16)),
+                   tdev(pool["page_table"]), tdev(pool["branch_len"]), tdev(pool["free"]),
+                   torch.tensor([pool["top"]], dtype=torch.int32, device=dev), inp.m)
+    k_new, v_new = (tdev(a.view(np.int16)) for a in kv_new)
+    reject_all = torch.full((inp.B,), -1, dtype=torch.int32, device=dev)
+
+    def kv_pair(r, i):
+        kv.append(k_new, v_new, stream)
+        kv.rollback(reject_all, stream)
+
+    with torch.cuda.stream(stream):
+        kv_pair(0, 0)
+    g_kv = capture(K, 0, kv_pair)
+    kv_ms = timer.median_ms([g_kv], n_rep) / K
+    if kv.errors(stream):
+        raise SystemExit(f"bench.py: KV append / rollback error flags {kv.errors(stream):#x}")
+    kv_bytes = 2 * 2 * inp.B * inp.m * inp.H_kv * inp.D * 2  # K and V rows read + written
+    res["kv_append_rollback"] = {
+        "us_per_pair": kv_ms * 1e3, "launches_per_pair": 3, "bytes": kv_bytes,
+        "achieved_gbs": kv_bytes / (kv_ms * 1e-3) / 1e9,
+        "note": "hpd_kv_append (m rows per branch) + hpd_kv_rollback (all rolled back) "
+                "on a pool of the workload's lengths; not part of the step metric"}
+
+    # ---- fork detection / child branches after the acceptance (reported beside
+    # the step): the step's argmax tokens, each page's first branch its layout
+    # branch, with the fork token emitted at its first position (always within
+    # the emitted span) and at its last emitted position
+    acc_np = acc.cpu().numpy()
+    fork_id = VOCAB - 1
+    fork_tok = np.where(argmax_np == fork_id, 0, argmax_np).astype(np.int32)
+    is_layout = np.zeros(inp.B, np.int32)
+    firsts = inp.branch_cu[:-1][np.diff(inp.branch_cu) > 0]
+    is_layout[firsts] = 1
+    for b in firsts:
+        fork_tok[b, 0] = fork_id
+        fork_tok[b, min(max(int(acc_np[b]), 0), inp.m - 1)] = fork_id
+    layout_pos = (inp.branch_prefix_len if inp.branch_prefix_len is not None
+                  else np.repeat(np.diff(inp.prefix_cu), np.diff(inp.branch_cu))).astype(np.int32)
+    layout_pos = np.maximum(layout_pos - inp.m, 0).astype(np.int32)
+    f_in = [tdev(a) for a in (fork_tok, acc_np, is_layout, layout_pos, inp.branch_cu,
+                               inp.branch_len, inp.page_table)]
+    f_cap = inp.B * (inp.m + 1)
+    f_state = {}
+
+    def fork_call(r, i):
+        f_state["out"] = H.fork_children(f_in[0], f_in[1], f_in[2], f_in[3], fork_id, f_in[4],
+                                         None, f_in[5], f_in[6], f_cap, stream)
+
+    with torch.cuda.stream(stream):
+        fork_call(0, 0)
+    torch.cuda.synchronize(dev)
+    n_children = int(f_state["out"]["new_B"].item()) - inp.B
+    g_fork = capture(K, 0, fork_call)
+    fork_ms = timer.median_ms([g_fork], n_rep) / K
+    res["fork_children"] = {
+        "us_per_call": fork_ms * 1e3, "children": n_children, "launches": 2,
+        "note": "hpd_fork_children over the step's branches: every page's layout branch "
+                "emits the fork token at its first and at its last emitted position; not "
+                "part of the step metric"}
+
+    # ---- the attention call on other layouts of the prefix and on the
+    # layout-branch workload (reported beside the step; one input replica)
+    def attn_call_us(inp_x):
+        op_x = H.BranchAttn(H.DeviceInputs.from_host(inp_x), stream)
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                op_x(stream)
+        torch.cuda.synchronize(dev)
+        g_x = capture(K, 0, lambda r, i: op_x(stream))
+        ms = timer.median_ms([g_x], n_rep) / K
+        if op_x.errors(stream):
+            raise SystemExit(f"bench.py: error flags {op_x.errors(stream):#x} on {inp_x.name}")
+        return ms * 1e3, H.hpd_branch_attn_launches(op_x.args)
+
+    runs_us, _ = attn_call_us(W.page_the_prefix(inp, seed=7000 + cid, runs=True))
+    scat_us, _ = attn_call_us(W.page_the_prefix(inp, seed=7000 + cid, runs=False))
+    res["paged_prefix"] = {
+        "us_per_call_consecutive_pages": runs_us, "us_per_call_scattered_pages": scat_us,
+        "contiguous_us_per_call": attn_ms * 1e3,
+        "note": "the same attention call with every page's prefix in the 16-token KV "
+                "pool through a prefix page table: in consecutive pool pages (one "
+                "prefill allocation) or scattered; one L2-warm input replica"}
+    lay = W.make_layout_config()
+    lay_us, lay_launch = attn_call_us(lay)
+    res["layout_branches"] = {
+        "workload": "8 pages, vision U[1024,3072], layout tokens U[64,512], each "
+                    "page's layout branch + U[4,24] content branches forked after "
+                    "a layout token (lognormal histories), m=4, Hq16/Hkv2, D128, "
+                    "paged prefix shared with the layout branch",
+        "us_per_call": lay_us, "launches": lay_launch,
+        "query_tokens_per_s": lay.B * lay.m / (lay_us * 1e-6),
+        "note": "attention call only, one L2-warm input replica"}
+    return res
+
+
+def run_ours(args, world, rank, local):
+    import torch
+    import torch.distributed as dist
+    from paper_2607_18839_gb300 import build as hpd_build
+    from paper_2607_18839_gb300 import hpd as H
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py: no CUDA device (the CUDA path has no CPU fallback)")
+    if world > 1:
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    hpd_build.build()
+    H.load()
+    stream = torch.cuda.Stream(device=dev)
+
+    head = measure_workload(args.workload, args, world, rank, dev, stream, H, headline=True)
+    others = [w for w in (args.also.split(",") if args.also else []) if w and w != args.workload]
+    per_config = {}
+    for w in others:
+        r = measure_workload(w, args, world, rank, dev, stream, H, headline=False)
+        per_config[w] = {
+            "config": step_config(w, world),
+            "value": r["value"], "ms_per_step": r["ms_per_step"], "roofline": r["roofline"],
+            "attention_only": r["attention_only"], "step_roofline": r["step_roofline"],
+            "e2e": r["e2e"], "kernel_us": r["kernel_us"], "cold_l2": r["cold_l2"],
+        }
+        del r
+        torch.cuda.empty_cache()
+
+    # ---- CPU baseline: the oracle on this host's cores (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, thr, sample = oracle_sample_run(head["inp"], head["logits_np"], head["drafts_np"],
+                                           args.cpu_seconds)
+        cpu = {"value": v, "unit": UNIT, "cores": thr, "kind": "oracle", "sample": sample}
+
+    if world > 1:
+        dist.destroy_process_group()
+    if rank != 0:
+        return None
+
+    K = args.steps
+    line = {
+        "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": max(args.warmup, 3), "ms_per_step": head["ms_per_step"],
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": step_config(args.workload, world),
+        "timing": {
+            "method": f"one CUDA graph of exactly {K} steps on the launch stream, replayed "
+                      f"{len(head['step_replays_ms'])} times, each replay bracketed by a "
+                      "barrier and a device synchronize and timed with CUDA events; "
+                      "ms_per_step = median replay / steps",
+            "replays_ms": head["step_replays_ms"],
+            "l2": head["l2"],
+            "per_kernel": "from graphs of back-to-back calls of each entry point after the "
+                          "timed region (median of the same number of replays); the attention "
+                          "call's kernels apportioned by in-graph timing markers",
+        },
+        "e2e": head["e2e"],
+        "gpu_launches": K * (head["n_launch"] + 1),
+        "roofline": head["roofline"],
+        "attention_only": head["attention_only"],
+        "step_roofline": head["step_roofline"],
+        "kernel_us": head["kernel_us"],
+        "accept": head["accept"],
+        "cold_l2": head["cold_l2"],
+        "per_config": per_config,
+        "kv_append_rollback": head["kv_append_rollback"],
+        "fork_children": head["fork_children"],
+        "paged_prefix": head["paged_prefix"],
+        "layout_branches": head["layout_branches"],
+        "context": PAPER_CONTEXT,
+        "host_wall_ms_per_step": head["wall_ms"] / K,
         "cpu_baseline": cpu,
-        "clocks": clk,
+        "clocks": head["clocks"],
     }
     return line
 
@@ -735,9 +876,7 @@ def run_reference(args, world, rank):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": f"{args.workload}: {W.CONFIG_DESCRIPTIONS[args.workload]}; acceptance "
-                               f"over bf16 logits [{inp.B} x {inp.m} x {VOCAB}]",
-                   "parallelism": "host CPU (OpenMP)"},
+        "config": step_config(args.workload, world),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -747,11 +886,15 @@ def run_reference(args, world, rank):
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20000)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--workload", choices=W.CONFIG_NAMES, default="c2")
-    ap.add_argument("--graph-steps", type=int, default=200, help="steps captured per CUDA graph")
+    ap.add_argument("--workload", choices=W.CONFIG_NAMES, default="c4",
+                    help="the headline workload (default: c4, the largest single-GPU preset)")
+    ap.add_argument("--also", default="c2,c3,c5",
+                    help="comma-separated workloads measured after the headline (per_config)")
+    ap.add_argument("--replays", type=int, default=5,
+                    help="timed replays of the K-step graph (the median is reported; >= 5)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle CPU-baseline budget")
     ap.add_argument("--ref-step-seconds", type=float, default=1.0,
                     help="oracle work per step of --impl reference")

@@ -200,9 +200,10 @@ hpd_status hpd_pmtp_accept(const void *logits, const int32_t *drafts, int B, int
  * field means what it means for hpd_branch_attn.
  *   - Nothing is allocated: no cudaMalloc, cudaFree or allocating library
  *     routine is called.
- *   - A shape whose hpd_branch_attn_workspace_size exceeds
- *     HPD_NOALLOC_WORKSPACE_BYTES is rejected with HPD_ERR_WORKSPACE before
- *     anything is enqueued.
+ *   - Every argument is checked as hpd_branch_attn checks it before
+ *     anything is enqueued; a refused call touches neither the array nor
+ *     the stream.  A shape whose hpd_branch_attn_workspace_size exceeds
+ *     HPD_NOALLOC_WORKSPACE_BYTES is refused with HPD_ERR_WORKSPACE.
  *   - The first call on a device looks up the array's device address
  *     (cudaGetSymbolAddress, with that device current); make that first call
  *     before any stream capture on the device.

@@ -8,7 +8,9 @@
 // the cluster size are taken in turn).  Each CTA streams its row with
 // 16-byte loads, reduces (value, index) over the CTA, and writes its token
 // to the output and into the leader CTA's shared memory (distributed shared
-// memory); after one cluster barrier the leader matches the drafts.
+// memory, written only after a cluster barrier shows that every CTA of the
+// cluster runs); after a second cluster barrier the leader matches the
+// drafts.
 #include <cooperative_groups.h>
 
 #include <climits>
@@ -128,6 +130,15 @@ __device__ __forceinline__ int row_argmax(const __nv_bfloat16 *row, int V, float
   return best.i == INT_MAX ? 0 : best.i;
 }
 
+// Split cluster barrier (every thread of every CTA of the cluster arrives
+// once, then waits for the phase).
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+}
+
 // grid (cluster size * B), cluster (cluster size, 1, 1): cluster = branch.
 __global__ void __launch_bounds__(kAcceptThreads)
     accept_cluster_kernel(const __nv_bfloat16 *__restrict__ logits,
@@ -142,13 +153,24 @@ __global__ void __launch_bounds__(kAcceptThreads)
   const int cs = static_cast<int>(cluster.num_blocks());
   const int b = blockIdx.x / cs;
   int *leader_tok = cluster.map_shared_rank(s_tok, 0);
+  // The leader's shared memory may be written only once the leader CTA is
+  // known to run: a split cluster barrier, whose arrive comes first and whose
+  // wait comes just before the first remote write, so that the first row's
+  // scan overlaps the other CTAs' start.
+  cluster_arrive_relaxed();
+  bool joined = false;
   for (int j = rank; j < m; j += cs) {
     const int tok = row_argmax(logits + (static_cast<size_t>(b) * m + j) * V, V, s_v, s_i, &s_none);
+    if (!joined) {  // uniform over the CTA
+      cluster_wait();
+      joined = true;
+    }
     if (threadIdx.x == 0) {
       out_tokens[static_cast<size_t>(b) * m + j] = tok;
       leader_tok[j] = tok;
     }
   }
+  if (!joined) cluster_wait();
   cluster.sync();  // every row's token is in the leader's shared memory
   if (rank == 0 && threadIdx.x == 0) {
     int k = 0;

@@ -197,6 +197,10 @@ cudaError_t launch_wait_selftest(uint32_t *err, uint64_t limit_ns, cudaStream_t 
 cudaError_t launch_suffix_stage(const AttnParams &p, const Plan &plan, cudaStream_t s);
 // Remember `e` for hpd_last_cuda_error() and return HPD_ERR_CUDA.
 hpd_status record_cuda_error(cudaError_t e);
+// Every host check of an hpd_branch_attn call except the workspace's:
+// scalars, required pointers and their alignment.  HPD_OK or the status the
+// call would return; touches no device state.
+hpd_status check_call_args(const hpd_branch_attn_args *a);
 // Leading workspace bytes that must be zero before a call (error word and
 // tickets); 0 if the scalars are invalid.
 size_t workspace_zero_bytes(const hpd_branch_attn_args *args);

@@ -132,6 +132,23 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
 
 hpd_status hpd::record_cuda_error(cudaError_t e) { return cuda_fail(e); }
 
+hpd_status hpd::check_call_args(const hpd_branch_attn_args *a) {
+  const hpd_status st = check_scalars(a);
+  if (st != HPD_OK) return st;
+  if (!a->q || !a->prefix_cu || !a->branch_cu || !a->k_cache || !a->v_cache || !a->page_table ||
+      !a->branch_len || !a->out)
+    return HPD_ERR_INVALID_ARG;
+  if (a->prefix_tokens > 0 && !a->prefix_page_table && (!a->prefix_k || !a->prefix_v))
+    return HPD_ERR_INVALID_ARG;
+  if (!aligned(a->q, 16) || !aligned(a->prefix_k, 16) || !aligned(a->prefix_v, 16) ||
+      !aligned(a->k_cache, 16) || !aligned(a->v_cache, 16) || !aligned(a->out, 16) ||
+      !aligned(a->lse, 4) || !aligned(a->prefix_cu, 4) || !aligned(a->branch_cu, 4) ||
+      !aligned(a->page_table, 4) || !aligned(a->branch_len, 4) ||
+      !aligned(a->branch_prefix_len, 4) || !aligned(a->prefix_page_table, 4))
+    return HPD_ERR_INVALID_ARG;
+  return HPD_OK;
+}
+
 size_t hpd::workspace_zero_bytes(const hpd_branch_attn_args *a) {
   if (check_scalars(a) != HPD_OK) return 0;
   return make_plan(a).off_opart;
@@ -177,19 +194,8 @@ hpd_status hpd_branch_attn(const hpd_branch_attn_args *a, hpd_stream_t stream) {
 
 hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t stream,
                                   void *const *ev) {
-  const hpd_status st = check_scalars(a);
+  const hpd_status st = hpd::check_call_args(a);
   if (st != HPD_OK) return st;
-  if (!a->q || !a->prefix_cu || !a->branch_cu || !a->k_cache || !a->v_cache || !a->page_table ||
-      !a->branch_len || !a->out)
-    return HPD_ERR_INVALID_ARG;
-  if (a->prefix_tokens > 0 && !a->prefix_page_table && (!a->prefix_k || !a->prefix_v))
-    return HPD_ERR_INVALID_ARG;
-  if (!aligned(a->q, 16) || !aligned(a->prefix_k, 16) || !aligned(a->prefix_v, 16) ||
-      !aligned(a->k_cache, 16) || !aligned(a->v_cache, 16) || !aligned(a->out, 16) ||
-      !aligned(a->lse, 4) || !aligned(a->prefix_cu, 4) || !aligned(a->branch_cu, 4) ||
-      !aligned(a->page_table, 4) || !aligned(a->branch_len, 4) ||
-      !aligned(a->branch_prefix_len, 4) || !aligned(a->prefix_page_table, 4))
-    return HPD_ERR_INVALID_ARG;
   const hpd::Plan pl = make_plan(a);
   if (!a->workspace || !aligned(a->workspace, kAlign) || a->workspace_bytes < pl.bytes)
     return HPD_ERR_WORKSPACE;

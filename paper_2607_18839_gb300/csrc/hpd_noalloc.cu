@@ -52,8 +52,12 @@ extern "C" hpd_status hpd_branch_attn_noalloc(const hpd_branch_attn_args *args,
   hpd_branch_attn_args a = *args;
   a.workspace = nullptr;
   a.workspace_bytes = 0;
+  // A call that is refused enqueues nothing, not even the clear of the
+  // shared array below: every argument check comes first.
+  const hpd_status st = hpd::check_call_args(&a);
+  if (st != HPD_OK) return st;
   const size_t need = hpd_branch_attn_workspace_size(&a);
-  if (need == 0) return hpd_branch_attn(&a, stream);  // reports the invalid scalars
+  if (need == 0) return HPD_ERR_INVALID_ARG;
   if (need > HPD_NOALLOC_WORKSPACE_BYTES) return HPD_ERR_WORKSPACE;
 
   void *scratch = nullptr;

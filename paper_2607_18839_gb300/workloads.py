@@ -406,6 +406,16 @@ CONFIG_DESCRIPTIONS = {
 }
 
 
+# Branches and P-MTP queries per branch of each preset.
+CONFIG_SHAPES = {"c1": (4, 1), "c2": (16, 4), "c3": (64, 4), "c4": (768, 8), "c5": (256, 4)}
+
+
+def config_shape(name: str) -> dict:
+    """{"B": branches, "m": queries per branch} of a preset, without drawing it."""
+    B, m = CONFIG_SHAPES[name]
+    return {"B": B, "m": m}
+
+
 def make_logits(B: int, m: int, V: int, seed: int) -> np.ndarray:
     """bf16 logits [B, m, V] drawn N(0, 1)."""
     rng = np.random.default_rng(seed)

@@ -123,6 +123,36 @@ def test_struct_layouts_match_the_header(tmp_path):
     assert got[3] == [ctypes.sizeof(F), F.fork_token.offset, F.cap.offset]
 
 
+def test_noalloc_limit_matches_the_header(tmp_path):
+    """The binding's NOALLOC_WORKSPACE_BYTES is the header macro's value."""
+    import shutil
+    import subprocess
+    if shutil.which("gcc") is None:
+        pytest.skip("no gcc")
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    src = tmp_path / "limit.c"
+    src.write_text('#include <stdio.h>\n#include "hpd.h"\n'
+                   'int main(void) { printf("%llu\\n", '
+                   '(unsigned long long)HPD_NOALLOC_WORKSPACE_BYTES); return 0; }\n')
+    exe = tmp_path / "limit"
+    subprocess.run(["gcc", "-I", os.path.join(root, "include"), str(src), "-o", str(exe)], check=True)
+    got = int(subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout)
+    assert got == hpd.NOALLOC_WORKSPACE_BYTES
+
+
+def test_noalloc_refuses_bad_arguments_before_enqueueing(lib):
+    # null pointers and a misaligned output are refused on the host, before
+    # the shared scratch array is touched (no GPU needed)
+    with pytest.raises(hpd.HpdError) as e:
+        hpd.hpd_branch_attn_noalloc(_args(), None)
+    assert e.value.status == 1
+    a = _args(q=4096, prefix_k=4096, prefix_v=4096, prefix_cu=4096, branch_cu=4096,
+              k_cache=4096, v_cache=4096, page_table=4096, branch_len=4096, out=4098)
+    with pytest.raises(hpd.HpdError) as e:
+        hpd.hpd_branch_attn_noalloc(a, None)
+    assert e.value.status == 1
+
+
 def _workload_args(inp):
     a = hpd.hpd_branch_attn_args()
     for k, v in dict(n_docs=inp.n_docs, B=inp.B, m=inp.m, H_q=inp.H_q, H_kv=inp.H_kv, D=inp.D,

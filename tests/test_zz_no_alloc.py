@@ -71,6 +71,12 @@ def test_noalloc_refuses_shapes_beyond_its_scratch(H):
                      num_pages=inp.num_pages, max_pages_per_branch=inp.max_pages,
                      prefix_tokens=inp.prefix_tokens).items():
         setattr(args, k, v)
+    # valid (small) device buffers: every argument check passes, so the size
+    # is what is refused, before anything is enqueued
+    buf = torch.zeros(4096, dtype=torch.uint8, device="cuda")
+    for f in ("q", "prefix_k", "prefix_v", "prefix_cu", "branch_cu", "k_cache", "v_cache",
+              "page_table", "branch_len", "out", "lse"):
+        setattr(args, f, buf.data_ptr())
     assert H.hpd_branch_attn_workspace_size(args) > H.NOALLOC_WORKSPACE_BYTES
     with pytest.raises(H.HpdError) as e:
         H.hpd_branch_attn_noalloc(args, None)
