@@ -284,8 +284,8 @@ hpd_status hpd_kv_rollback(const hpd_kv_args *args, const int32_t *accepted_len,
  * *new_B = the new branch count, or -1 with HPD_DEVERR_FORK_CAP in the
  * workspace error word when it would exceed cap (the outputs are then not
  * written).  workspace: 256-byte aligned, >= 4 * (65 + n_docs) bytes, word 0
- * the error word (cleared by the caller).  Two launches (a one-CTA scan, then
- * the copy of the old branches' arrays), asynchronous on `stream`.
+ * the error word (cleared by the caller).  One launch (B + n_docs up to
+ * 11,998; two launches beyond), asynchronous on `stream`.
  * ------------------------------------------------------------------------ */
 typedef struct {
   const int32_t *out_tokens;         /* [B][m] (hpd_pmtp_accept) */

@@ -12,7 +12,16 @@
 // prefix position layout_pos[b] + i.  Every emitted fork token spawns one
 // child with prefix length layout_pos[b] + i + 1.  The new branch arrays keep
 // each page's old branches in order and append its children after them, in
-// (parent, index) order.  One CTA scans, so the placement is deterministic.
+// (parent, index) order; the placement comes from a scan in branch order, so
+// it is deterministic.
+//
+// One launch (B + n_docs up to kMaxFused): every CTA counts every branch's
+// children and scans the counts in its own shared memory (the outputs never
+// alias the inputs, so no CTA waits for another), then writes its share of
+// the new arrays.  With c_b the children of branch b and pre_b their
+// exclusive sum over branches, page d's old branches move by pre at its first
+// branch, and branch b's children start at new index branch_cu[d+1] + pre_b.
+// Larger calls take two launches (one CTA scans page by page, then many copy).
 #include <algorithm>
 
 #include "common.cuh"
@@ -21,6 +30,8 @@ namespace hpd {
 namespace {
 
 constexpr int kForkThreads = 1024;
+constexpr int kFusedThreads = 256;
+constexpr int kMaxFused = 12000;  // B + n_docs + 2 ints of shared memory (48,000 bytes)
 
 // Block-wide exclusive scan of one value per thread; total to *total.
 __device__ __forceinline__ int fork_scan(int x, int *ws, int *total) {
@@ -150,6 +161,113 @@ __global__ void __launch_bounds__(kForkThreads) fork_kernel(hpd_fork_args a) {
   }
 }
 
+// The whole fork step in one launch (see the top of the file).
+__global__ void __launch_bounds__(kFusedThreads) fork_fused_kernel(hpd_fork_args a) {
+  extern __shared__ int s_dyn[];
+  int *pre = s_dyn;                 // [B + 1] children of branches before b
+  int *cu = s_dyn + a.B + 1;        // [n_docs + 1] branch_cu
+  __shared__ int warp_sums[kFusedThreads / 32];
+  __shared__ int s_bad, s_total;
+  uint32_t *err = static_cast<uint32_t *>(a.workspace);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  pdl_wait();  // whatever ran before on the stream has finished
+  if (tid == 0) {
+    s_bad = a.branch_cu[0] != 0 || a.branch_cu[a.n_docs] != a.B;
+    s_total = 0;
+  }
+  for (int d = tid; d <= a.n_docs; d += kFusedThreads) cu[d] = a.branch_cu[d];
+  __syncthreads();
+  for (int d = tid; d < a.n_docs; d += kFusedThreads)
+    if (cu[d] > cu[d + 1]) s_bad = 1;
+  __syncthreads();
+  if (s_bad) {  // nothing written but the error
+    if (blockIdx.x == 0 && tid == 0) {
+      atomicOr(err, HPD_DEVERR_BRANCH_CU);
+      *a.new_B = -1;
+    }
+    return;
+  }
+  for (int b0 = 0; b0 < a.B; b0 += kFusedThreads) {
+    const int b = b0 + tid;
+    const int f = b < a.B ? n_forks(a, b) : 0;
+    int incl = f;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    if (lane == 31) warp_sums[warp] = incl;
+    __syncthreads();
+    int woff = 0;
+    for (int w = 0; w < warp; ++w) woff += warp_sums[w];
+    if (b < a.B) pre[b] = s_total + woff + incl - f;
+    __syncthreads();
+    if (tid == kFusedThreads - 1) s_total += woff + incl;
+    __syncthreads();
+  }
+  if (tid == 0) pre[a.B] = s_total;
+  __syncthreads();
+  const int n_children = s_total;
+  if (a.B + n_children > a.cap) {
+    if (blockIdx.x == 0 && tid == 0) {
+      atomicOr(err, HPD_DEVERR_FORK_CAP);
+      *a.new_B = -1;
+    }
+    return;
+  }
+  // page of branch b: the largest d with cu[d] <= b
+  auto doc = [&](int b) {
+    int lo = 0, hi = a.n_docs;
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (cu[mid] <= b) lo = mid; else hi = mid;
+    }
+    return lo;
+  };
+  const size_t stride = static_cast<size_t>(gridDim.x) * kFusedThreads;
+  const size_t t0 = static_cast<size_t>(blockIdx.x) * kFusedThreads + tid;
+  if (t0 == 0) *a.new_B = a.B + n_children;
+  for (size_t d = t0; d <= static_cast<size_t>(a.n_docs); d += stride)
+    a.new_branch_cu[d] = cu[d] + pre[cu[d]];
+  for (size_t b = t0; b < static_cast<size_t>(a.B); b += stride) {
+    const int ib = static_cast<int>(b), d = doc(ib);
+    const size_t nb = b + pre[cu[d]];
+    a.new_parent[nb] = ib;
+    a.new_branch_len[nb] = a.branch_len[b];
+    a.new_branch_prefix_len[nb] = a.branch_prefix_len ? a.branch_prefix_len[b] : -1;
+    const int f = pre[ib + 1] - pre[ib];
+    if (f > 0) {  // its children: after the page's old branches, in index order
+      int slot = cu[d + 1] + pre[ib];
+      const int n = a.accepted_len[b];
+      const int e = n < 0 ? 0 : min(n + 1, a.m);
+      for (int i = 0; i < e; ++i) {
+        if (a.out_tokens[b * a.m + i] != a.fork_token) continue;
+        a.new_parent[slot] = -1 - ib;
+        a.new_branch_len[slot] = 0;
+        a.new_branch_prefix_len[slot] = a.layout_pos[b] + i + 1;
+        ++slot;
+      }
+    }
+  }
+  for (size_t i = t0; i < static_cast<size_t>(a.B) * a.max_pages; i += stride) {
+    const int b = static_cast<int>(i / a.max_pages);
+    const size_t nb = b + pre[cu[doc(b)]];
+    a.new_page_table[nb * a.max_pages + i % a.max_pages] = a.page_table[i];
+  }
+  // the children's page-table rows are all -1
+  for (size_t i = t0; i < static_cast<size_t>(n_children) * a.max_pages; i += stride) {
+    // child number c (in new-index order over pages) -> its new index
+    const int c = static_cast<int>(i / a.max_pages);
+    int lo = 0, hi = a.n_docs;  // the page holding child c: largest d with pre[cu[d]] <= c
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (pre[cu[mid]] <= c) lo = mid; else hi = mid;
+    }
+    const size_t slot = cu[lo + 1] + c;  // children of page lo after its old branches
+    a.new_page_table[slot * a.max_pages + i % a.max_pages] = -1;
+  }
+}
+
 // The old branches' arrays, moved past the children of earlier pages (many
 // CTAs, after fork_kernel on the same stream; nothing when it failed).
 __global__ void fork_copy_kernel(hpd_fork_args a) {
@@ -187,12 +305,23 @@ extern "C" hpd_status hpd_fork_children(const hpd_fork_args *a, hpd_stream_t str
   if (a->workspace_bytes < static_cast<size_t>(64 + a->n_docs + 1) * sizeof(int))
     return HPD_ERR_WORKSPACE;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  hpd::fork_kernel<<<1, hpd::kForkThreads, 0, s>>>(*a);
-  if (a->B > 0) {
+  cudaError_t e = cudaSuccess;
+  if (static_cast<long long>(a->B) + a->n_docs + 2 <= hpd::kMaxFused) {
+    // one launch; it may start while the previous kernel on the stream
+    // finishes (it waits for it before reading anything)
     const long long n = static_cast<long long>(a->B) * a->max_pages;
-    const int grid = static_cast<int>(std::min<long long>((n + 255) / 256, 1216));
-    hpd::fork_copy_kernel<<<grid, 256, 0, s>>>(*a);
+    const int grid = static_cast<int>(std::max<long long>(1, std::min<long long>((n + 2047) / 2048, 64)));
+    const size_t smem = sizeof(int) * (static_cast<size_t>(a->B) + a->n_docs + 2);
+    e = hpd::launch_kernel(true, hpd::fork_fused_kernel, dim3(grid), dim3(hpd::kFusedThreads), smem,
+                           s, *a);
+  } else {
+    hpd::fork_kernel<<<1, hpd::kForkThreads, 0, s>>>(*a);
+    if (a->B > 0) {
+      const long long n = static_cast<long long>(a->B) * a->max_pages;
+      const int grid = static_cast<int>(std::min<long long>((n + 255) / 256, 1216));
+      hpd::fork_copy_kernel<<<grid, 256, 0, s>>>(*a);
+    }
+    e = cudaGetLastError();
   }
-  const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? HPD_OK : hpd::record_cuda_error(e);
 }
