@@ -716,7 +716,9 @@ def measure_workload(name, args, world, rank, dev, stream, H, headline):
     g_fork = capture(K, 0, fork_call)
     fork_ms = timer.median_ms([g_fork], n_rep) / K
     res["fork_children"] = {
-        "us_per_call": fork_ms * 1e3, "children": n_children, "launches": 2,
+        "us_per_call": fork_ms * 1e3, "children": n_children,
+        # one launch up to B + n_docs = 11,998 (the shared-memory scan), two beyond
+        "launches": 1 if inp.B + inp.n_docs <= 11998 else 2,
         "note": "hpd_fork_children over the step's branches: every page's layout branch "
                 "emits the fork token at its first and at its last emitted position; not "
                 "part of the step metric"}

@@ -14,8 +14,9 @@
 //
 // Both stages split their key range into chunks and write, per chunk, the
 // normalised partial output O_s (fp32) and its log-sum-exp lse_s (natural
-// log; -inf when the chunk holds no visible key).  merge_accept.cu combines
-// them.
+// log; -inf when the chunk holds no visible key).  The suffix stage combines
+// them: for each branch, the last of its suffix CTAs to finish merges every
+// slot of the branch's rows by log-sum-exp and writes out / lse.
 #include <atomic>
 
 #include "common.cuh"
