@@ -274,8 +274,10 @@ def step_config(name, world):
         "workload": f"{name}: {inp_desc}; acceptance over bf16 logits "
                     f"[{cfg['B']} x {cfg['m']} x {VOCAB}]",
         "query_tokens_per_step": cfg["B"] * cfg["m"],
-        "step": "hpd_branch_attn (shared prefix + private suffix + merge) then hpd_pmtp_accept "
-                "(acceptance inside the step)",
+        "step": "hpd_decode_step: hpd_branch_attn (shared prefix + private suffix + merge) and "
+                "hpd_pmtp_accept (acceptance inside the step; it reads only the logits and drafts, "
+                "so it runs beside the attention when the attention's grid leaves SMs idle, "
+                "else after it)",
         "parallelism": f"dp{world} (independent pages per GPU, no collective)",
     }
 
@@ -373,9 +375,11 @@ def measure_workload(name, args, world, rank, dev, stream, H, headline):
         H.hpd_pmtp_accept(logits[r].data_ptr(), drafts.data_ptr(), inp.B, inp.m, VOCAB,
                           out_tokens.data_ptr(), acc.data_ptr(), sh)
 
-    def step(r, ev=None):
-        attn(r, ev)
-        accept(r)
+    # one step: hpd_decode_step (the attention, and the acceptance beside it
+    # when the attention leaves SMs idle, else after it)
+    def step(r):
+        H.hpd_decode_step(argsets[r], logits[r].data_ptr(), drafts.data_ptr(), VOCAB,
+                          out_tokens.data_ptr(), acc.data_ptr(), sh)
 
     # ---- warm-up (eager), also sets the kernels' function attributes
     with torch.cuda.stream(stream):
@@ -436,24 +440,25 @@ def measure_workload(name, args, world, rank, dev, stream, H, headline):
     kernel_ms = {nm: attn_ms * span[k] / sum(span) for k, nm in enumerate(attn_names)}
     kernel_ms[ACCEPT] = acc_ms
 
-    # ---- cold L2: before each step a write of twice the L2 size evicts
-    # everything; events around the step alone
+    # ---- cold L2: before each step (and before each attention call alone) a
+    # write of twice the L2 size evicts everything; events around the call
     flush = torch.empty(2 * l2, dtype=torch.uint8, device=dev)
     n_cold = max(5, min(20, K))
-    ev_cold = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
-                torch.cuda.Event(enable_timing=True)) for _ in range(n_cold)]
+    ev_cold = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(n_cold)]
     torch.cuda.synchronize(dev)
     with torch.cuda.stream(stream):
-        for i, (e0, e1, e2) in enumerate(ev_cold):
+        for i, (e0, e1, e2, e3) in enumerate(ev_cold):
             flush.fill_(i & 0xff)
             e0.record(stream)
-            attn(i % R)
+            step(i % R)
             e1.record(stream)
-            accept(i % R)
+            flush.fill_((i + 1) & 0xff)
             e2.record(stream)
+            attn(i % R)
+            e3.record(stream)
     torch.cuda.synchronize(dev)
-    cold_step_ms = statistics.median(e0.elapsed_time(e2) for e0, _, e2 in ev_cold)
-    cold_attn_ms = statistics.median(e0.elapsed_time(e1) for e0, e1, _ in ev_cold)
+    cold_step_ms = statistics.median(e0.elapsed_time(e1) for e0, e1, _, _ in ev_cold)
+    cold_attn_ms = statistics.median(e2.elapsed_time(e3) for _, _, e2, e3 in ev_cold)
     del flush
 
     # ---- end to end: pinned host inputs in, results out, every step.  Each
@@ -540,9 +545,8 @@ def measure_workload(name, args, world, rank, dev, stream, H, headline):
                 stream.wait_event(ev_in)
                 if i >= 2:
                     stream.wait_event(out_done[i - 2])  # the slot's results were read out
-                H.hpd_branch_attn(slot_args(s_i, r), sh)
-                H.hpd_pmtp_accept(sl["lg"].data_ptr(), sl["dr"].data_ptr(), inp.B, inp.m, VOCAB,
-                                  sl["tok"].data_ptr(), sl["acc"].data_ptr(), sh)
+                H.hpd_decode_step(slot_args(s_i, r), sl["lg"].data_ptr(), sl["dr"].data_ptr(),
+                                  VOCAB, sl["tok"].data_ptr(), sl["acc"].data_ptr(), sh)
                 comp[i] = torch.cuda.Event()
                 comp[i].record(stream)
                 with torch.cuda.stream(d2h_s):
@@ -627,6 +631,7 @@ def measure_workload(name, args, world, rank, dev, stream, H, headline):
                           "t_roofline_us": t_step_roof * 1e6,
                           "frac": t_step_roof / (ms_step * 1e-3)},
         "kernel_us": {k: v * 1e3 for k, v in kernel_ms.items()},
+        "accept_beside_attention": H.hpd_decode_step_concurrent(argsets[0]) == 1,
         "accept": {"us_per_call": acc_us, "bytes": per[ACCEPT]["bytes"],
                    "achieved_gbs": per[ACCEPT]["bytes"] / (acc_us * 1e-6) / 1e9,
                    "frac_of_measured_hbm":
@@ -784,6 +789,7 @@ def run_ours(args, world, rank, local):
             "value": r["value"], "ms_per_step": r["ms_per_step"], "roofline": r["roofline"],
             "attention_only": r["attention_only"], "step_roofline": r["step_roofline"],
             "e2e": r["e2e"], "kernel_us": r["kernel_us"], "cold_l2": r["cold_l2"],
+            "accept_beside_attention": r["accept_beside_attention"],
         }
         del r
         torch.cuda.empty_cache()
@@ -826,6 +832,7 @@ def run_ours(args, world, rank, local):
         "kernel_us": head["kernel_us"],
         "accept": head["accept"],
         "cold_l2": head["cold_l2"],
+        "accept_beside_attention": head["accept_beside_attention"],
         "per_config": per_config,
         "kv_append_rollback": head["kv_append_rollback"],
         "fork_children": head["fork_children"],

@@ -186,6 +186,37 @@ hpd_status hpd_pmtp_accept(const void *logits, const int32_t *drafts, int B, int
                            int32_t *out_tokens, int32_t *accepted_len, hpd_stream_t stream);
 
 /*
+ * One branch-decode step (Algorithm 1: the model step, then verification):
+ * hpd_branch_attn(args) and hpd_pmtp_accept over logits [B][m][V] and drafts
+ * [B][m] (B = args->B, m = args->m), with exactly the results of the two
+ * calls made in that order on `stream`, and the same argument checks and
+ * errors (nothing is enqueued when either call's arguments are refused).
+ *
+ * The acceptance reads only logits and drafts, none of the attention's
+ * results, so the two need not run one after the other.  When the attention
+ * kernel leaves SMs idle for part of its run (fewer than two work units per
+ * SM: its persistent grid is smaller than the SM count, as on a one-page
+ * step, or its last round of whole units leaves SMs idle) the acceptance
+ * runs on those SMs while the attention runs: it is launched on a second
+ * stream owned by the library,
+ * forked from `stream` and joined back to it with events, so the step stays
+ * ordered on `stream` (work enqueued on `stream` afterwards waits for both)
+ * and can be captured in a CUDA graph.  Otherwise the acceptance follows the
+ * attention on `stream`.  The second stream and its two events are created
+ * on the first call made outside stream capture on each device (a call
+ * inside capture before then runs the two in order).  Calls from several
+ * host threads take a lock while they enqueue.
+ */
+hpd_status hpd_decode_step(const hpd_branch_attn_args *args, const void *logits,
+                           const int32_t *drafts, int V, int32_t *out_tokens,
+                           int32_t *accepted_len, hpd_stream_t stream);
+
+/* 1 when hpd_decode_step would run the acceptance concurrently with the
+ * attention for these host scalars (device pointers are not read), 0 when
+ * in order, -1 for invalid scalars or an unavailable device. */
+int hpd_decode_step_concurrent(const hpd_branch_attn_args *args);
+
+/*
  * hpd_branch_attn for callers that cannot allocate device memory.  The
  * paper has no counterpart to this entry point.
  *

@@ -4,6 +4,7 @@
 // here touches device data.
 #include <cmath>
 #include <cstdint>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -127,6 +128,54 @@ hpd::Plan make_plan(const hpd_branch_attn_args *a) {
   pl.bytes = align_up(pl.off_order + n_units * sizeof(int));
   return pl;
 }
+
+hpd_status check_accept_args(const void *logits, const int32_t *drafts, int B, int m, int V,
+                             const int32_t *out_tokens, const int32_t *accepted_len) {
+  if (!logits || !drafts || !out_tokens || !accepted_len) return HPD_ERR_INVALID_ARG;
+  if (B < 1 || m < 1 || V < 1) return HPD_ERR_INVALID_ARG;
+  if (m > 64) return HPD_ERR_UNSUPPORTED;
+  if (!aligned(logits, 2) || !aligned(drafts, 4) || !aligned(out_tokens, 4) ||
+      !aligned(accepted_len, 4))
+    return HPD_ERR_INVALID_ARG;
+  return HPD_OK;
+}
+
+// SM count of the current device (cached per device); 0 when unavailable.
+int device_sms(int *dev_out) {
+  static int sms[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (sms[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    sms[dev] = n;
+  }
+  if (dev_out) *dev_out = dev;
+  return sms[dev];
+}
+
+// The attention kernel leaves SMs idle for part of its run: with fewer
+// than two work units per SM its persistent CTAs (one per SM) either do not
+// fill the GPU or finish their last round of whole units at different times.
+// The acceptance then runs beside it on the idle SMs.  With more units per
+// SM the dynamic scheduler keeps every SM busy until near the end and the
+// two run in order.
+constexpr int kConcurrentUnitsPerSm = 2;
+bool step_concurrent(const hpd::Plan &pl, const hpd_branch_attn_args *a, int sms) {
+  if (!pl.use_tc || sms <= 0) return false;
+  const long long units = static_cast<long long>(pl.tiles_max) * a->H_kv * pl.S_p;
+  return units < static_cast<long long>(kConcurrentUnitsPerSm) * sms;
+}
+
+// Per device: the second stream of hpd_decode_step and its fork / join
+// events, created on the first call outside stream capture.
+struct StepStreams {
+  std::mutex mu;
+  bool ready = false;
+  cudaStream_t side = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+};
+StepStreams g_step[64];
 
 }  // namespace
 
@@ -282,15 +331,75 @@ hpd_status hpd_branch_attn_marked(const hpd_branch_attn_args *a, hpd_stream_t st
 
 hpd_status hpd_pmtp_accept(const void *logits, const int32_t *drafts, int B, int m, int V,
                            int32_t *out_tokens, int32_t *accepted_len, hpd_stream_t stream) {
-  if (!logits || !drafts || !out_tokens || !accepted_len) return HPD_ERR_INVALID_ARG;
-  if (B < 1 || m < 1 || V < 1) return HPD_ERR_INVALID_ARG;
-  if (m > 64) return HPD_ERR_UNSUPPORTED;
-  if (!aligned(logits, 2) || !aligned(drafts, 4) || !aligned(out_tokens, 4) ||
-      !aligned(accepted_len, 4))
-    return HPD_ERR_INVALID_ARG;
+  const hpd_status st = check_accept_args(logits, drafts, B, m, V, out_tokens, accepted_len);
+  if (st != HPD_OK) return st;
   const cudaError_t e =
       hpd::launch_accept(static_cast<const __nv_bfloat16 *>(logits), drafts, B, m, V, out_tokens,
                          accepted_len, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? HPD_OK : cuda_fail(e);
+}
+
+int hpd_decode_step_concurrent(const hpd_branch_attn_args *args) {
+  if (check_scalars(args) != HPD_OK) return -1;
+  const int sms = device_sms(nullptr);
+  if (sms <= 0) return -1;
+  return step_concurrent(make_plan(args), args, sms) ? 1 : 0;
+}
+
+hpd_status hpd_decode_step(const hpd_branch_attn_args *a, const void *logits,
+                           const int32_t *drafts, int V, int32_t *out_tokens,
+                           int32_t *accepted_len, hpd_stream_t stream) {
+  hpd_status st = hpd::check_call_args(a);
+  if (st != HPD_OK) return st;
+  st = check_accept_args(logits, drafts, a->B, a->m, V, out_tokens, accepted_len);
+  if (st != HPD_OK) return st;
+  const hpd::Plan pl = make_plan(a);
+  if (!a->workspace || !aligned(a->workspace, kAlign) || a->workspace_bytes < pl.bytes)
+    return HPD_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  auto accept_on = [&](cudaStream_t t) {
+    return hpd::launch_accept(static_cast<const __nv_bfloat16 *>(logits), drafts, a->B, a->m, V,
+                              out_tokens, accepted_len, t);
+  };
+  int dev = 0;
+  const int sms = device_sms(&dev);
+  if (!step_concurrent(pl, a, sms)) {
+    st = hpd_branch_attn(a, stream);
+    if (st != HPD_OK) return st;
+    const cudaError_t e = accept_on(s);
+    return e == cudaSuccess ? HPD_OK : cuda_fail(e);
+  }
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(s, &cap);
+  if (e != cudaSuccess) return cuda_fail(e);
+  StepStreams &ss = g_step[dev];
+  std::lock_guard<std::mutex> lock(ss.mu);
+  if (!ss.ready && cap == cudaStreamCaptureStatusNone) {
+    e = cudaStreamCreateWithFlags(&ss.side, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ss.fork, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ss.join, cudaEventDisableTiming);
+    if (e != cudaSuccess) return cuda_fail(e);
+    ss.ready = true;
+  }
+  if (!ss.ready) {  // first call inside a capture: in order
+    st = hpd_branch_attn(a, stream);
+    if (st != HPD_OK) return st;
+    e = accept_on(s);
+    return e == cudaSuccess ? HPD_OK : cuda_fail(e);
+  }
+  // fork: the second stream waits for everything enqueued on `stream` so
+  // far; the attention is enqueued first, then the acceptance beside it
+  e = cudaEventRecord(ss.fork, s);
+  if (e != cudaSuccess) return cuda_fail(e);
+  e = cudaStreamWaitEvent(ss.side, ss.fork, 0);
+  if (e != cudaSuccess) return cuda_fail(e);
+  st = hpd_branch_attn(a, stream);
+  cudaError_t ea = st == HPD_OK ? accept_on(ss.side) : cudaSuccess;
+  // join (also after a failed launch, so that a capture is never left forked)
+  e = cudaEventRecord(ss.join, ss.side);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(s, ss.join, 0);
+  if (st != HPD_OK) return st;
+  if (ea != cudaSuccess) return cuda_fail(ea);
   return e == cudaSuccess ? HPD_OK : cuda_fail(e);
 }
 

@@ -24,9 +24,11 @@ DEVERR = {0x1: "PREFIX_CU", 0x2: "BRANCH_CU", 0x4: "BRANCH_LEN", 0x8: "PAGE_ID",
 
 # Every entry point declared in include/hpd.h.
 EXPORTS = ("hpd_branch_attn_workspace_size", "hpd_workspace_init", "hpd_branch_attn",
-           "hpd_branch_attn_launches", "hpd_branch_attn_kernel_name", "hpd_branch_attn_marked", "hpd_pmtp_accept", "hpd_read_errors", "hpd_status_string", "hpd_last_cuda_error",
-           "hpd_version", "hpd_branch_attn_noalloc", "hpd_wait_selftest", "hpd_kv_append",
-           "hpd_kv_rollback", "hpd_fork_children")
+           "hpd_branch_attn_launches", "hpd_branch_attn_kernel_name", "hpd_branch_attn_marked",
+           "hpd_pmtp_accept", "hpd_decode_step", "hpd_decode_step_concurrent",
+           "hpd_read_errors", "hpd_status_string", "hpd_last_cuda_error", "hpd_version",
+           "hpd_branch_attn_noalloc", "hpd_wait_selftest", "hpd_kv_append", "hpd_kv_rollback",
+           "hpd_fork_children")
 
 # Scratch bytes built into libhpd for hpd_branch_attn_noalloc.
 NOALLOC_WORKSPACE_BYTES = 32 << 20
@@ -112,6 +114,10 @@ def load(path: str = LIB_PATH):
                                            ctypes.POINTER(ctypes.c_void_p)]
     lib.hpd_pmtp_accept.restype = I
     lib.hpd_pmtp_accept.argtypes = [P, P, I, I, I, P, P, P]
+    lib.hpd_decode_step.restype = I
+    lib.hpd_decode_step.argtypes = [ctypes.POINTER(hpd_branch_attn_args), P, P, I, P, P, P]
+    lib.hpd_decode_step_concurrent.restype = I
+    lib.hpd_decode_step_concurrent.argtypes = [ctypes.POINTER(hpd_branch_attn_args)]
     lib.hpd_read_errors.restype = I
     lib.hpd_read_errors.argtypes = [P, ctypes.POINTER(ctypes.c_uint32), P]
     lib.hpd_status_string.restype = ctypes.c_char_p
@@ -188,6 +194,20 @@ def hpd_pmtp_accept(logits_ptr, drafts_ptr, B, m, V, out_tokens_ptr, accepted_le
     _check("hpd_pmtp_accept", load().hpd_pmtp_accept(logits_ptr, drafts_ptr, B, m, V,
                                                      out_tokens_ptr, accepted_len_ptr,
                                                      stream_handle))
+
+
+def hpd_decode_step(args: hpd_branch_attn_args, logits_ptr, drafts_ptr, V, out_tokens_ptr,
+                    accepted_len_ptr, stream_handle) -> None:
+    """hpd_branch_attn(args) and hpd_pmtp_accept (B = args.B, m = args.m) as
+    one step; the acceptance runs beside the attention when the attention
+    leaves SMs idle (see include/hpd.h)."""
+    _check("hpd_decode_step", load().hpd_decode_step(ctypes.byref(args), logits_ptr, drafts_ptr,
+                                                     V, out_tokens_ptr, accepted_len_ptr,
+                                                     stream_handle))
+
+
+def hpd_decode_step_concurrent(args: hpd_branch_attn_args) -> int:
+    return int(load().hpd_decode_step_concurrent(ctypes.byref(args)))
 
 
 def hpd_read_errors(workspace_ptr: int, stream_handle) -> int:
@@ -337,6 +357,14 @@ class BranchAttn:
         else:
             hpd_branch_attn_marked(self.args, _stream_handle(stream),
                                    [int(e.cuda_event) for e in events])
+        return self.out, self.lse
+
+    def step(self, logits, drafts, out_tokens, accepted_len, stream=None):
+        """Enqueue one decode step: this attention call and the acceptance of
+        ``logits`` (bf16 [B, m, V]) against ``drafts`` (int32 [B, m]) into
+        ``out_tokens`` (int32 [B, m]) and ``accepted_len`` (int32 [B])."""
+        hpd_decode_step(self.args, _ptr(logits), _ptr(drafts), int(logits.shape[-1]),
+                        _ptr(out_tokens), _ptr(accepted_len), _stream_handle(stream))
         return self.out, self.lse
 
     def errors(self, stream=None) -> int:

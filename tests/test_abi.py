@@ -91,6 +91,15 @@ def test_accept_rejects_bad_arguments_before_launch(lib):
     assert e.value.status == 2
 
 
+def test_decode_step_rejects_bad_arguments_before_launch(lib):
+    # the attention's arguments are checked first, then the acceptance's;
+    # either refusal returns before anything reaches a device
+    with pytest.raises(hpd.HpdError) as e:
+        hpd.hpd_decode_step(_args(), 16, 16, 100, 16, 16, None)
+    assert e.value.status == 1
+    assert hpd.hpd_decode_step_concurrent(_args(D=80)) == -1
+
+
 def test_struct_layouts_match_the_header(tmp_path):
     """sizeof / offsetof of the C structs, compiled from include/hpd.h, equal
     the ctypes mirrors of the binding."""
