@@ -148,3 +148,45 @@ def test_step_refuses_bad_arguments_before_enqueueing(hpd):
                                tok.data_ptr(), acc.data_ptr(), h) == 1
     torch.cuda.synchronize()
     assert bool((op.out.float() == 3.0).all())
+
+
+def special_logits(B, m, V, seed):
+    """Logits with the cases the argmax must get exactly right: ties (the
+    lowest index wins), -0 against +0, NaN (never wins), rows of NaN and -inf
+    (the first -inf wins), a row of NaN only (token 0), and maxima at the
+    last index and around index 8192."""
+    rng = np.random.default_rng(seed)
+    x = rng.integers(-4, 5, size=(B, m, V)).astype(np.float32)  # many ties
+    x[0, 0, :] = 0.0
+    x[0, 0, 7::9] = -0.0
+    x[0, 1, :] = np.nan
+    x[0, 1, 3] = -np.inf
+    x[0, 1, 11] = -np.inf
+    x[0, 2, :] = np.nan                      # all NaN -> token 0
+    x[1, :, 5::13] = np.nan                  # NaN mixed with values
+    x[2, 0, :] = -np.inf
+    x[3, 0, V - 1] = 100.0
+    if V > 8192:
+        x[3, 1, 8192] = 100.0
+        x[3, 2, 8191] = 100.0
+    return W.f32_to_bf16_bits(x)
+
+
+@pytest.mark.parametrize("name,V_", [("c4", 4096), ("c4", 20001), ("c2", 32000)])
+def test_step_acceptance_special_values(hpd, name, V_):
+    inp = W.make_config(name)
+    logits = special_logits(inp.B, inp.m, V_, seed=V_)
+    ref_tok0, _ = oracle.pmtp_accept(logits, np.zeros((inp.B, inp.m), np.int32))
+    drafts = W.mix_drafts(ref_tok0, V_, 0.7, seed=V_ + 1)
+    ref_tok, ref_acc = oracle.pmtp_accept(logits, drafts)
+    assert ref_tok[0, 2] == 0 and ref_tok[0, 1] == 3 and ref_tok[2, 0] == 0
+    lg = torch.from_numpy(logits.view(np.int16)).cuda().view(torch.bfloat16)
+    dr = torch.from_numpy(drafts).cuda()
+    op = hpd.BranchAttn(hpd.DeviceInputs.from_host(inp))
+    tok = torch.full((inp.B, inp.m), -7, dtype=torch.int32, device="cuda")
+    acc = torch.full((inp.B,), -7, dtype=torch.int32, device="cuda")
+    op.step(lg, dr, tok, acc)
+    torch.cuda.synchronize()
+    assert op.errors() == 0
+    np.testing.assert_array_equal(tok.cpu().numpy(), ref_tok)
+    np.testing.assert_array_equal(acc.cpu().numpy(), ref_acc)
