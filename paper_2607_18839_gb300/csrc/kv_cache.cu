@@ -15,6 +15,11 @@
 // those of branches 0..b-1, whatever the launch order.  All or nothing: when
 // the stack is short or a branch would outgrow its table row, nothing
 // changes and the error word gets HPD_DEVERR_POOL / HPD_DEVERR_BRANCH_LEN.
+// Up to kScanThreads branches the scan is one pass (each thread keeps its
+// branch's values); beyond, a first pass checks the capacity and a second
+// assigns.  Each kernel is launched with programmatic dependent launch: it
+// waits for its predecessor on the stream before touching any state, and
+// lets its successor start launching right away.
 #include <algorithm>
 
 #include "common.cuh"
@@ -72,11 +77,42 @@ __global__ void __launch_bounds__(kScanThreads) kv_append_alloc_kernel(KvArgs a)
   __shared__ int warp_sums[33];
   __shared__ int s_bad, s_need;
   const int tid = threadIdx.x;
+  pdl_wait();     // the previous kernel's lengths, tables and stack
+  pdl_trigger();  // the copy may launch; it waits for this kernel
   if (tid == 0) {
     s_bad = 0;
     s_need = 0;
   }
   __syncthreads();
+  if (a.B <= kScanThreads) {  // one pass
+    const int b = tid;
+    int need = 0, L = 0;
+    if (b < a.B) {
+      L = a.branch_len[b];
+      if (L < 0 || L + a.m > a.max_pages * kPage) atomicOr(&s_bad, 1);
+      else need = pages_of(L + a.m) - pages_of(L);
+    }
+    int total;
+    const int before = block_scan(need, warp_sums, &total);  // orders the s_bad writes
+    const int top = *a.free_top;
+    if (s_bad || total > top || top > a.num_pages) {
+      if (tid == 0) {
+        atomicOr(a.err, s_bad ? HPD_DEVERR_BRANCH_LEN : HPD_DEVERR_POOL);
+        *a.done = 0;
+      }
+      return;
+    }
+    if (b < a.B) {
+      int32_t *row = a.page_table + static_cast<size_t>(b) * a.max_pages;
+      for (int i = 0; i < need; ++i) row[pages_of(L) + i] = a.free_pages[top - total + before + i];
+      a.branch_len[b] = L + a.m;
+    }
+    if (tid == 0) {
+      *a.free_top = top - total;
+      *a.done = 1;
+    }
+    return;
+  }
   // capacity check and total pages needed
   for (int b0 = 0; b0 < a.B; b0 += kScanThreads) {
     const int b = b0 + tid;
@@ -127,6 +163,8 @@ __global__ void __launch_bounds__(kScanThreads) kv_append_alloc_kernel(KvArgs a)
 // Pass 2 of the append: copy the new rows, 16 bytes per thread, when pass 1
 // succeeded (*done; otherwise nothing was allocated and nothing is written).
 __global__ void kv_append_copy_kernel(KvArgs a, int rows_total) {
+  pdl_wait();  // the allocation
+  pdl_trigger();
   if (*reinterpret_cast<volatile int32_t *>(a.done) == 0) return;
   const int vec_per_row = a.D / 8;  // 16-byte vectors of one (row, head)
   const long long n = static_cast<long long>(rows_total) * a.H_kv * vec_per_row;
@@ -155,6 +193,8 @@ __global__ void __launch_bounds__(kScanThreads)
   __shared__ int warp_sums[33];
   __shared__ int s_bad, s_free;
   const int tid = threadIdx.x;
+  pdl_wait();  // the previous kernel's lengths, tables, stack and accepted lengths
+  pdl_trigger();
   if (tid == 0) {
     s_bad = 0;
     s_free = 0;
@@ -165,6 +205,36 @@ __global__ void __launch_bounds__(kScanThreads)
     const int keep = n < 0 ? 0 : min(n + 1, a.m);
     return L - a.m + keep;
   };
+  if (a.B <= kScanThreads) {  // one pass
+    const int b = tid;
+    int fr = 0, L = 0, Ln = 0;
+    if (b < a.B) {
+      L = a.branch_len[b];
+      if (L < a.m || L > a.max_pages * kPage) {
+        atomicOr(&s_bad, 1);
+      } else {
+        Ln = new_len(b, L);
+        fr = pages_of(L) - pages_of(Ln);
+      }
+    }
+    int total;
+    const int before = block_scan(fr, warp_sums, &total);  // orders the s_bad writes
+    const int top = *a.free_top;
+    if (s_bad || top < 0 || top + total > a.num_pages) {
+      if (tid == 0) atomicOr(a.err, s_bad ? HPD_DEVERR_BRANCH_LEN : HPD_DEVERR_POOL);
+      return;
+    }
+    if (b < a.B) {
+      int32_t *row = a.page_table + static_cast<size_t>(b) * a.max_pages;
+      for (int i = 0; i < fr; ++i) {
+        a.free_pages[top + before + i] = row[pages_of(Ln) + i];
+        row[pages_of(Ln) + i] = -1;
+      }
+      a.branch_len[b] = Ln;
+    }
+    if (tid == 0) *a.free_top = top + total;
+    return;
+  }
   for (int b0 = 0; b0 < a.B; b0 += kScanThreads) {
     const int b = b0 + tid;
     int fr = 0;
@@ -244,11 +314,13 @@ hpd_status hpd_kv_append(const hpd_kv_args *args, hpd_stream_t stream) {
     return HPD_ERR_INVALID_ARG;
   if (args->B == 0) return HPD_OK;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  hpd::kv_append_alloc_kernel<<<1, hpd::kScanThreads, 0, s>>>(k);
+  cudaError_t e = hpd::launch_kernel(true, hpd::kv_append_alloc_kernel, dim3(1),
+                                     dim3(hpd::kScanThreads), 0, s, k);
   const long long vecs = static_cast<long long>(args->B) * args->m * args->H_kv * (args->D / 8);
   const int grid = static_cast<int>(std::min<long long>((vecs + 255) / 256, 152 * 8));
-  hpd::kv_append_copy_kernel<<<grid, 256, 0, s>>>(k, args->B * args->m);
-  const cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess)
+    e = hpd::launch_kernel(true, hpd::kv_append_copy_kernel, dim3(grid), dim3(256), 0, s, k,
+                           args->B * args->m);
   return e == cudaSuccess ? HPD_OK : hpd::record_cuda_error(e);
 }
 
@@ -259,9 +331,9 @@ hpd_status hpd_kv_rollback(const hpd_kv_args *args, const int32_t *accepted_len,
   if (st != HPD_OK) return st;
   if (!accepted_len) return HPD_ERR_INVALID_ARG;
   if (args->B == 0) return HPD_OK;
-  hpd::kv_rollback_kernel<<<1, hpd::kScanThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-      k, accepted_len);
-  const cudaError_t e = cudaGetLastError();
+  const cudaError_t e =
+      hpd::launch_kernel(true, hpd::kv_rollback_kernel, dim3(1), dim3(hpd::kScanThreads), 0,
+                         reinterpret_cast<cudaStream_t>(stream), k, accepted_len);
   return e == cudaSuccess ? HPD_OK : hpd::record_cuda_error(e);
 }
 

@@ -60,6 +60,15 @@ def test_c5_like_branches():
     _run(lengths, m=4, H=8, D=128, pages=2500, max_pages=48, steps=4, seed=11)
 
 
+def test_c4_like_branches():
+    # 768 branches and 1024 (the largest one-pass scan)
+    rng = np.random.default_rng(2)
+    lengths = np.clip(np.round(rng.lognormal(4.5, 0.8, 768)), 1, 1024).astype(np.int32)
+    _run(lengths, m=8, H=2, D=128, pages=8000, max_pages=70, steps=3, seed=16)
+    lengths = rng.integers(0, 40, size=1024).astype(np.int32)
+    _run(lengths, m=4, H=2, D=64, pages=5000, max_pages=4, steps=2, seed=17)
+
+
 def test_many_branches_two_scan_chunks_d64():
     rng = np.random.default_rng(1)
     lengths = rng.integers(2, 70, size=1500).astype(np.int32)
