@@ -205,7 +205,9 @@ hpd_status hpd_pmtp_accept(const void *logits, const int32_t *drafts, int B, int
  * attention on `stream`.  The second stream and its two events are created
  * on the first call made outside stream capture on each device (a call
  * inside capture before then runs the two in order).  Calls from several
- * host threads take a lock while they enqueue.
+ * host threads take a lock while they enqueue.  The second stream is shared
+ * by every call on the device, so the acceptances of steps issued on
+ * different streams run one after another.
  */
 hpd_status hpd_decode_step(const hpd_branch_attn_args *args, const void *logits,
                            const int32_t *drafts, int V, int32_t *out_tokens,
