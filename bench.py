@@ -276,8 +276,8 @@ def step_config(name, world):
         "query_tokens_per_step": cfg["B"] * cfg["m"],
         "step": "hpd_decode_step: hpd_branch_attn (shared prefix + private suffix + merge) and "
                 "hpd_pmtp_accept (acceptance inside the step; it reads only the logits and drafts, "
-                "so it runs beside the attention when the attention's grid leaves SMs idle, "
-                "else after it)",
+                "so it runs beside the attention when the attention has fewer than two work units "
+                "per SM and leaves SMs idle, else after it)",
         "parallelism": f"dp{world} (independent pages per GPU, no collective)",
     }
 
