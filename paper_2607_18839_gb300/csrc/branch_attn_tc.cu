@@ -535,13 +535,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint64_t dk0 = smem_desc_sw128(sbase + L::kK, 16, 1024);
     // S[col] = Q (TMEM slot qs) K^T of global block jg: A from TMEM, 16
     // dimensions (8 columns) per MMA; B = K, K-major in shared memory
+    // (one lane, elected once per group, issues the group's MMAs and commits)
+    const bool issuer = elect_one();
     auto issue_qk = [&](int qs, int jg, uint32_t col) {
       const uint64_t kd = dk0 + (((jg % L::kKStages) * L::kTileBytes) >> 4);
+      if (issuer) {
 #pragma unroll
-      for (int kk = 0; kk < D / 16; ++kk) {
-        const uint32_t off = ((kk >> 2) * L::kChunkBytes + (kk & 3) * 32) >> 4;
-        mma_ts(tmem + col, tmem + L::col_q(qs) + kk * 8, kd + off, idesc_qk, kk > 0);
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = ((kk >> 2) * L::kChunkBytes + (kk & 3) * 32) >> 4;
+          mma_ts_one(tmem + col, tmem + L::col_q(qs) + kk * 8, kd + off, idesc_qk, kk > 0);
+        }
       }
+      __syncwarp();
+    };
+    auto commit = [&](uint64_t &b) {
+      if (issuer) mma_commit_one(bar(b));
+      __syncwarp();
     };
     // O (+)= P V of global block jg, P in TMEM at column pcol: one
     // N = D MMA per 16 keys.  V is MN-major (D contiguous): 64-column swizzle
@@ -550,10 +559,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint64_t dv0 = smem_desc_sw128(sbase + L::kV, L::kChunkBytes, 1024);
     auto issue_pv = [&](int jg, bool first, uint32_t pcol) {
       const uint64_t vd = dv0 + (((jg % L::kVStages) * L::kTileBytes) >> 4);
+      if (issuer) {
 #pragma unroll
-      for (int kk = 0; kk < kBlk / 16; ++kk)
-        mma_ts(tmem + L::kColO, tmem + pcol + kk * 8, vd + ((kk * 16 * 128) >> 4), idesc_pv,
-               (!first || kk > 0) ? 1u : 0u);
+        for (int kk = 0; kk < kBlk / 16; ++kk)
+          mma_ts_one(tmem + L::kColO, tmem + pcol + kk * 8, vd + ((kk * 16 * 128) >> 4), idesc_pv,
+                     (!first || kk > 0) ? 1u : 0u);
+      }
+      __syncwarp();
     };
     auto wait = [&](uint64_t &b, int parity) {
       if (!wait_bar(b, parity)) return false;
@@ -575,9 +587,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       // O last held unit x.unit - 1, whose epilogue must have read it
       if (x.first && x.unit >= 1 && !wait(sh.o_empty, (x.unit - 1) & 1)) return false;
       issue_pv(x.jg, x.first, L::col_s(s));
-      mma_commit(bar(sh.pv_done));
-      mma_commit(bar(sh.v_empty[sv]));
-      if (x.last) mma_commit(bar(sh.o_full));
+      commit(sh.pv_done);
+      commit(sh.v_empty[sv]);
+      if (x.last) commit(sh.o_full);
       return true;
     };
     int jbase = 0;
@@ -596,9 +608,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int jg = jbase + j, s = jg & 1, sk = jg % L::kKStages;
         if (!(ok = wait(sh.k_full[sk], (jg / L::kKStages) & 1))) break;
         issue_qk(qs, jg, L::col_s(s));
-        mma_commit(bar(sh.s_full[s]));
-        mma_commit(bar(sh.k_empty[sk]));
-        if (j == nb - 1) mma_commit(bar(sh.q_empty[qs]));
+        commit(sh.s_full[s]);
+        commit(sh.k_empty[sk]);
+        if (j == nb - 1) commit(sh.q_empty[qs]);
         if (has_pend && !(ok = do_pv(pend))) break;
         pend = Pending{jg, k, j == 0, j == nb - 1};
         has_pend = true;
