@@ -48,6 +48,11 @@ __device__ __forceinline__ float softmax_half_tmem(uint32_t s_addr, int h, int l
   const bool all_full = __all_sync(0xffffffffu, lo == 0 && hi == kH);
   uint32_t v[kH];
   float mx = NEG_INF;
+  // A positive scale keeps the order of the scores, so the maximum can be
+  // taken over the raw scores and an invisible score can simply become -inf
+  // in place (its exponential is then 0): one select per score instead of a
+  // visibility test in both loops below.
+  const bool raw = sl2 > 0.f;
   if (!all_empty) {
     tmem_ld32(s_addr + h * kH, v);
     tmem_ld32(s_addr + h * kH + 32, v + 32);
@@ -55,8 +60,20 @@ __device__ __forceinline__ float softmax_half_tmem(uint32_t s_addr, int h, int l
     float mx8[8];
 #pragma unroll
     for (int a = 0; a < 8; ++a) mx8[a] = NEG_INF;
-    if (all_full && sl2 > 0.f) {
-      // raw scores: a positive scale keeps the order
+    if (raw) {
+      if (!all_full) {
+        // bit c of vis: column c of this half is visible
+        auto below = [](int n) -> uint64_t {
+          return n <= 0 ? 0ull : n >= 64 ? ~0ull : (1ull << n) - 1ull;
+        };
+        const uint64_t vis = below(hi) & ~below(lo);
+        const uint32_t vis0 = static_cast<uint32_t>(vis), vis1 = static_cast<uint32_t>(vis >> 32);
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          v[c] = (vis0 & (1u << c)) ? v[c] : 0xff800000u;
+          v[c + 32] = (vis1 & (1u << c)) ? v[c + 32] : 0xff800000u;
+        }
+      }
 #pragma unroll
       for (int c = 0; c < kH; c += 16)
 #pragma unroll
@@ -75,7 +92,7 @@ __device__ __forceinline__ float softmax_half_tmem(uint32_t s_addr, int h, int l
     }
     mx = fmax3(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(mx8[3], mx8[4], mx8[5]),
                fmaxf(mx8[6], mx8[7]));
-    if (all_full && sl2 > 0.f) mx *= sl2;
+    if (raw) mx *= sl2;
   }
   mx = xchg(mx);
   const float m_new = mx > m_run + kRescaleLog2 ? mx : m_run;
@@ -93,7 +110,7 @@ __device__ __forceinline__ float softmax_half_tmem(uint32_t s_addr, int h, int l
     float2 sum4[4];
 #pragma unroll
     for (int a = 0; a < 4; ++a) sum4[a] = make_float2(0.f, 0.f);
-    if (all_full) {
+    if (all_full || raw) {
 #pragma unroll
       for (int ch = 0; ch < 2; ++ch) {
 #pragma unroll

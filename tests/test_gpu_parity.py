@@ -81,6 +81,15 @@ SMALL = {
                                                  128, seed=42, branch_prefix_len=[200, 7, 150, 50, 0]),
     "g5_d64_warp_mma_prefix": lambda: W.build_inputs([129], [4], [1, 2, 3, 100], 2, 10, 2, 64,
                                                      seed=43),
+    # m G = 64: row tiles of two branches, whose private pages fill one half of
+    # each suffix block each (lengths L = s + m of 8, 64, 65, 128, 308 keys:
+    # empty halves, segment ends, several blocks), plus one-branch tiles
+    "two_branch_tiles": lambda: W.build_inputs(
+        [700, 130, 0], [5, 2, 3], [0, 1, 56, 57, 120, 200, 8, 300, 63, 64], 8, 16, 2, 128,
+        seed=49),
+    "two_branch_tiles_d64_fork": lambda: W.build_inputs(
+        [400, 90], [4, 2], [3, 250, 60, 0, 17, 129], 4, 16, 1, 64, seed=50,
+        branch_prefix_len=[400, 0, 128, 399, 90, 1]),
     # many pages with one branch each, long prefixes split across CTAs
     "many_pages_split_prefix": lambda: W.build_inputs([1000 + 37 * i for i in range(12)], [1] * 12,
                                                       [5 * i for i in range(12)], 4, 16, 2, 128,
