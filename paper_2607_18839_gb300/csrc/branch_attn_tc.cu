@@ -580,10 +580,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     };
     Pending pend{0, 0, false, false};
     bool has_pend = false;
-    auto do_pv = [&](const Pending &x) -> bool {
-      const int s = x.jg & 1, sv = x.jg % L::kVStages;
-      if (!wait(sh.p_full[s], (x.jg >> 1) & 1) || !wait(sh.v_full[sv], (x.jg / L::kVStages) & 1))
-        return false;
+    // V of block x.jg and K of block jn (the next Q K^T) are tested while
+    // the warp waits for P of block x.jg, so that their shared-memory round
+    // trips overlap; only phases not yet complete are waited for again.
+    // k_next: K of block jn has landed.
+    auto do_pv = [&](const Pending &x, int jn, bool &k_next) -> bool {
+      const int s = x.jg & 1, sv = x.jg % L::kVStages, sk = jn % L::kKStages;
+      uint32_t r = mbar_try_test2(bar(sh.p_full[s]), (x.jg >> 1) & 1, bar(sh.v_full[sv]),
+                                  (x.jg / L::kVStages) & 1, bar(sh.k_full[sk]),
+                                  (jn / L::kKStages) & 1);
+      r = __shfl_sync(0xffffffffu, r, 0);
+      k_next = (r & 4u) != 0;
+      if (!(r & 1u) && !wait_bar(sh.p_full[s], (x.jg >> 1) & 1)) return false;
+      if (!(r & 2u) && !wait_bar(sh.v_full[sv], (x.jg / L::kVStages) & 1)) return false;
+      tc_fence_after();
       // O last held unit x.unit - 1, whose epilogue must have read it
       if (x.first && x.unit >= 1 && !wait(sh.o_empty, (x.unit - 1) & 1)) return false;
       issue_pv(x.jg, x.first, L::col_s(s));
@@ -593,7 +603,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       return true;
     };
     int jbase = 0;
-    bool ok = true;
+    bool ok = true, k_ready = false;
     for (int k = 0; ok; ++k) {
       const int slot = k & 1;
       if (!(ok = wait(sh.meta_full[slot], (k >> 1) & 1))) break;
@@ -606,18 +616,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!(ok = wait(sh.q_full[qs], (k >> 1) & 1))) break;
       for (int j = 0; j < nb; ++j) {
         const int jg = jbase + j, s = jg & 1, sk = jg % L::kKStages;
-        if (!(ok = wait(sh.k_full[sk], (jg / L::kKStages) & 1))) break;
+        if (!k_ready && !(ok = wait(sh.k_full[sk], (jg / L::kKStages) & 1))) break;
         issue_qk(qs, jg, L::col_s(s));
         commit(sh.s_full[s]);
         commit(sh.k_empty[sk]);
         if (j == nb - 1) commit(sh.q_empty[qs]);
-        if (has_pend && !(ok = do_pv(pend))) break;
+        k_ready = false;
+        if (has_pend && !(ok = do_pv(pend, jg + 1, k_ready))) break;
         pend = Pending{jg, k, j == 0, j == nb - 1};
         has_pend = true;
       }
       jbase += nb;
     }
-    if (ok && has_pend) ok = do_pv(pend);
+    if (ok && has_pend) ok = do_pv(pend, jbase, k_ready);
     if (!ok && lane == 0) set_abort(sh, p.err);
   } else {
     // --------------------------------------------------------- softmax --

@@ -45,6 +45,28 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// A try_wait on phase (b0, p0), which may suspend the thread for a while
+// until the phase completes, preceded by non-blocking tests of (b1, p1) and
+// (b2, p2) whose shared-memory round trips overlap it.  Bit i of the result
+// is set when phase i has completed (acquire, like a wait).
+__device__ __forceinline__ uint32_t mbar_try_test2(uint32_t b0, uint32_t p0, uint32_t b1,
+                                                   uint32_t p1, uint32_t b2, uint32_t p2) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred a, b, c;\n\t.reg .b32 x, y, z;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 b, [%3], %4;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 c, [%5], %6;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 a, [%1], %2;\n\t"
+      "selp.b32 x, 1, 0, a;\n\t"
+      "selp.b32 y, 2, 0, b;\n\t"
+      "selp.b32 z, 4, 0, c;\n\t"
+      "or.b32 x, x, y;\n\t"
+      "or.b32 %0, x, z;\n\t}"
+      : "=r"(r)
+      : "r"(b0), "r"(p0), "r"(b1), "r"(p1), "r"(b2), "r"(p2)
+      : "memory");
+  return r;
+}
 // try_wait that lets the thread sleep until the phase completes, for at most
 // about `ns` nanoseconds, so that waiting warps leave the issue slots of
 // their SM sub-partition to the warps that compute.
