@@ -124,7 +124,6 @@ struct TcLayout {
 
 struct __align__(8) TcShared {
   uint64_t meta_full[2], meta_empty[2];
-  uint64_t q_full[2], q_empty[2];  // Q rows in TMEM, per unit slot
   uint64_t k_full[kMaxRing], v_full[kMaxRing];
   uint64_t k_empty[kMaxRing], v_empty[kMaxRing];
   uint64_t s_full[2], p_full[2];  // per S buffer
@@ -185,7 +184,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                           const __grid_constant__ CUtensorMap tm_kc,
                           const __grid_constant__ CUtensorMap tm_vc,
                           const __grid_constant__ CUtensorMap tm_k8,
-                          const __grid_constant__ CUtensorMap tm_v8, const AttnParams p) {
+                          const __grid_constant__ CUtensorMap tm_v8,
+                          const __grid_constant__ CUtensorMap tm_q, const AttnParams p) {
   using L = TcLayout<D>;
   extern __shared__ uint8_t smem_raw[];
   __shared__ TcShared sh;
@@ -216,8 +216,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(bar(sh.meta_empty[s]), kMetaConsumers);
       mbar_init(bar(sh.s_full[s]), 1);
       mbar_init(bar(sh.p_full[s]), kSoftmaxWarps);
-      mbar_init(bar(sh.q_full[s]), kSoftmaxWarps);
-      mbar_init(bar(sh.q_empty[s]), 1);
     }
     mbar_init(bar(sh.pv_done), 1);
     mbar_init(bar(sh.o_full), 1);
@@ -413,9 +411,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 0 || warp == kVWarp) {
     // ------------------------------------------------------- producers --
     // The whole warp runs this loop with warp-uniform values; one elected
-    // lane issues each copy.  Warp 0: Q and K; warp kVWarp: V.
+    // lane issues each copy.  Warp 0: Q and K; warp kVWarp: V.  The K ring
+    // carries each unit's Q tile ahead of its K blocks: ring entry jbase + k
+    // is unit k's Q, entry jg + k + 1 the K of global block jg.
     const bool is_k = warp == 0;
     if (lane == 0) {
+      prefetch_tmap(&tm_q);
       prefetch_tmap(&tm_k);
       prefetch_tmap(&tm_v);
       prefetch_tmap(&tm_kc);
@@ -490,17 +491,26 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       };
+      if (is_k) {  // the unit's Q tile: tokens [tok0, tok0 + 128 / G), heads of KV head g
+        const int e = jbase + k, s = e % L::kKStages;
+        if (e >= L::kKStages && !(ok = wait_bar(sh.k_empty[s], ((e / L::kKStages) - 1) & 1)))
+          break;
+        mbar_arrive_expect_tx_elect(bar(sh.k_full[s]), L::kTileBytes);
+        for (int c = 0; c < L::kChunks; ++c)
+          tma_load_3d_elect(sbase + L::kK + s * L::kTileBytes + c * L::kChunkBytes, &tm_q,
+                            bar(sh.k_full[s]), c * 64, g * G, M.tok0);
+        issued_k = e + 1;
+      }
       for (int j = 0; j < nb; ++j) {
         const int jg = jbase + j;
         const int pid = prefix_pid(blk_lo + j);
         if (is_k) {
-          const int s = jg % L::kKStages;
-          if (jg >= L::kKStages &&
-              !(ok = wait_bar(sh.k_empty[s], ((jg / L::kKStages) - 1) & 1)))
+          const int e = jg + k + 1, s = e % L::kKStages;
+          if (e >= L::kKStages && !(ok = wait_bar(sh.k_empty[s], ((e / L::kKStages) - 1) & 1)))
             break;
           load_block(blk_lo + j, pid, sbase + L::kK + s * L::kTileBytes, bar(sh.k_full[s]), &tm_k,
                      &tm_kc, &tm_k8);
-          issued_k = jg + 1;
+          issued_k = e + 1;
         } else {
           const int s = jg % L::kVStages;
           if (jg >= L::kVStages &&
@@ -537,8 +547,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // dimensions (8 columns) per MMA; B = K, K-major in shared memory
     // (one lane, elected once per group, issues the group's MMAs and commits)
     const bool issuer = elect_one();
-    auto issue_qk = [&](int qs, int jg, uint32_t col) {
-      const uint64_t kd = dk0 + (((jg % L::kKStages) * L::kTileBytes) >> 4);
+    auto issue_qk = [&](int qs, int sk, uint32_t col) {
+      const uint64_t kd = dk0 + ((sk * L::kTileBytes) >> 4);
       if (issuer) {
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
@@ -584,13 +594,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     // the warp waits for P of block x.jg, so that their shared-memory round
     // trips overlap; only phases not yet complete are waited for again.
     // k_next: K of block jn has landed.
+    // (jn: ring entry of the next K block, or -1 when the next entry is a Q)
     auto do_pv = [&](const Pending &x, int jn, bool &k_next) -> bool {
-      const int s = x.jg & 1, sv = x.jg % L::kVStages, sk = jn % L::kKStages;
+      const int s = x.jg & 1, sv = x.jg % L::kVStages;
+      const int kb = jn >= 0 ? bar(sh.k_full[jn % L::kKStages]) : bar(sh.v_full[sv]);
+      const int kp = jn >= 0 ? (jn / L::kKStages) & 1 : (x.jg / L::kVStages) & 1;
       uint32_t r = mbar_try_test2(bar(sh.p_full[s]), (x.jg >> 1) & 1, bar(sh.v_full[sv]),
-                                  (x.jg / L::kVStages) & 1, bar(sh.k_full[sk]),
-                                  (jn / L::kKStages) & 1);
+                                  (x.jg / L::kVStages) & 1, kb, kp);
       r = __shfl_sync(0xffffffffu, r, 0);
-      k_next = (r & 4u) != 0;
+      k_next = jn >= 0 && (r & 4u) != 0;
       if (!(r & 1u) && !wait_bar(sh.p_full[s], (x.jg >> 1) & 1)) return false;
       if (!(r & 2u) && !wait_bar(sh.v_full[sv], (x.jg / L::kVStages) & 1)) return false;
       tc_fence_after();
@@ -612,23 +624,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (!valid) break;
       if (lane == 0) mbar_arrive(bar(sh.meta_empty[slot]));
-      const int qs = k & 1;
-      if (!(ok = wait(sh.q_full[qs], (k >> 1) & 1))) break;
+      // the unit's Q: from its K-ring entry into TMEM slot qs (the copy runs
+      // in order with the MMAs: unit k - 2's Q K^T are done with the slot)
+      const int qs = k & 1, qe = jbase + k, sq = qe % L::kKStages;
+      if (!(ok = wait(sh.k_full[sq], (qe / L::kKStages) & 1))) break;
+      if (issuer) {
+        const uint64_t qd = dk0 + ((sq * L::kTileBytes) >> 4);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk)
+          tmem_cp_128x256b(tmem + L::col_q(qs) + kk * 8,
+                           qd + (((kk >> 2) * L::kChunkBytes + (kk & 3) * 32) >> 4));
+      }
+      __syncwarp();
+      commit(sh.k_empty[sq]);
+      k_ready = false;
       for (int j = 0; j < nb; ++j) {
-        const int jg = jbase + j, s = jg & 1, sk = jg % L::kKStages;
-        if (!k_ready && !(ok = wait(sh.k_full[sk], (jg / L::kKStages) & 1))) break;
-        issue_qk(qs, jg, L::col_s(s));
+        const int jg = jbase + j, s = jg & 1, ke = jg + k + 1, sk = ke % L::kKStages;
+        if (!k_ready && !(ok = wait(sh.k_full[sk], (ke / L::kKStages) & 1))) break;
+        issue_qk(qs, sk, L::col_s(s));
         commit(sh.s_full[s]);
         commit(sh.k_empty[sk]);
-        if (j == nb - 1) commit(sh.q_empty[qs]);
         k_ready = false;
-        if (has_pend && !(ok = do_pv(pend, jg + 1, k_ready))) break;
+        if (has_pend && !(ok = do_pv(pend, j + 1 < nb ? ke + 1 : -1, k_ready))) break;
         pend = Pending{jg, k, j == 0, j == nb - 1};
         has_pend = true;
       }
       jbase += nb;
     }
-    if (ok && has_pend) ok = do_pv(pend, jbase, k_ready);
+    if (ok && has_pend) ok = do_pv(pend, -1, k_ready);
     if (!ok && lane == 0) set_abort(sh, p.err);
   } else {
     // --------------------------------------------------------- softmax --
@@ -648,9 +671,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       int g, split, nb, blk_lo, nP, lim_p, ps, last;
       size_t pair;
     };
-    // Reads unit k's metadata (slot k & 1), releases the slot, and copies the
-    // row's half of Q (D / 2 dimensions) into TMEM slot k & 1 once unit k - 2's
-    // Q K^T MMAs are done with it; false on timeout / abort.
+    // Reads unit k's metadata (slot k & 1) and releases the slot (the unit's
+    // Q reaches TMEM through the K ring and the MMA warp); false on timeout /
+    // abort.
     auto begin_unit = [&](int k, Row &R) -> bool {
       const int slot = k & 1;
       if (!wait_bar(sh.meta_full[slot], (k >> 1) & 1)) return false;
@@ -671,33 +694,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         R.pair = static_cast<size_t>(token) * p.H_q + R.g * G + r_in % G;
       }
       __syncwarp();
-      if (!R.unit) return true;
-      if (lane == 0) mbar_arrive(bar(sh.meta_empty[slot]));
-      uint32_t w[D / 4];
-      if (R.valid) {
-        const uint4 *src = reinterpret_cast<const uint4 *>(p.q + R.pair * D + h * (D / 2));
-#pragma unroll
-        for (int i = 0; i < D / 16; ++i) {
-          const uint4 x = __ldg(src + i);
-          w[4 * i] = x.x;
-          w[4 * i + 1] = x.y;
-          w[4 * i + 2] = x.z;
-          w[4 * i + 3] = x.w;
-        }
-      } else {
-#pragma unroll
-        for (int i = 0; i < D / 4; ++i) w[i] = 0u;
-      }
-      if (k >= 2 && !wait_bar(sh.q_empty[slot], ((k >> 1) - 1) & 1)) return false;
-      tc_fence_after();
-      if constexpr (D == 128)
-        tmem_st32(t_lane + L::col_q(slot) + h * (D / 4), w);
-      else
-        tmem_st16(t_lane + L::col_q(slot) + h * (D / 4), w);
-      tmem_st_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(bar(sh.q_full[slot]));
+      if (R.unit && lane == 0) mbar_arrive(bar(sh.meta_empty[slot]));
       return true;
     };
     const uint32_t o_col = L::kColO + h * (D / 2);
@@ -849,8 +846,9 @@ template <int D>
 cudaError_t launch_tc(const AttnParams &p, bool overlap, cudaStream_t s) {
   using L = TcLayout<D>;
   static_assert(L::kDynSmem + sizeof(TcShared) <= 227 * 1024, "shared memory");
-  CUtensorMap tk, tv, tkc, tvc, tk8, tv8;
+  CUtensorMap tk, tv, tkc, tvc, tk8, tv8, tq;
   cudaError_t e = tc::make_prefix_maps(p, &tk, &tv);
+  if (e == cudaSuccess) e = tc::make_q_map(p, &tq);
   if (e == cudaSuccess) e = tc::make_page_map(&tkc, p.k_cache, D, p.H_kv, p.num_pages);
   if (e == cudaSuccess) e = tc::make_page_map(&tvc, p.v_cache, D, p.H_kv, p.num_pages);
   const int run = std::min(kPagesPerBlock, p.num_pages);  // box never longer than the pool
@@ -877,7 +875,7 @@ cudaError_t launch_tc(const AttnParams &p, bool overlap, cudaStream_t s) {
   }
   const dim3 grid(static_cast<unsigned>(std::min(p.n_units, sms[dev & 63])), 1, 1);
   return launch_kernel(overlap, branch_attn_tc_kernel<D>, grid, dim3(kThreads), L::kDynSmem, s,
-                       tk, tv, tkc, tvc, tk8, tv8, p);
+                       tk, tv, tkc, tvc, tk8, tv8, tq, p);
 }
 
 }  // namespace

@@ -157,6 +157,13 @@ __device__ __forceinline__ void mma_ts_one(uint32_t d_tmem, uint32_t a_tmem, uin
       "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// TMEM (128 lanes x 8 columns at d_tmem) <- a 128-row x 32-byte matrix in
+// shared memory (descriptor s_desc, as for tcgen05.mma): row r lands in lane
+// r, in the layout an A operand read from TMEM has.  Asynchronous; ordered
+// with the tcgen05.mma instructions the same thread issues.
+__device__ __forceinline__ void tmem_cp_128x256b(uint32_t d_tmem, uint64_t s_desc) {
+  asm volatile("tcgen05.cp.cta_group::1.128x256b [%0], %1;" ::"r"(d_tmem), "l"(s_desc) : "memory");
+}
 __device__ __forceinline__ void mma_commit_one(uint32_t bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)

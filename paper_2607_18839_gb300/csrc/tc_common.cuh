@@ -203,8 +203,14 @@ inline cudaError_t make_page_map(CUtensorMap *map, const void *base, int D, int 
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-// Maps of Q (box: 64 columns x G heads x 128/G tokens = one 128-row tile)
-// and of the prefix K / V (box: 64 columns x 1 head x 128 keys).
+// Map of Q ([B m][H_q][D]): one box is 64 columns x G heads x 128 / G
+// tokens, i.e. one 128-row tile of stacked query rows (row = token x G +
+// head within the KV group) in the layout of a 128-key K block; rows past
+// the last token read zeros.
+inline cudaError_t make_q_map(const AttnParams &p, CUtensorMap *tq) {
+  return make_map(tq, p.q, p.D, p.H_q, static_cast<uint64_t>(p.rows_total), 64, p.G, kRows / p.G);
+}
+
 // K and V maps of the contiguous prefix ([tokens][H_kv][D], one KV head x
 // 128 keys x 64 columns per box); the paged cache stands in when there is
 // no prefix at all (the maps are then never used).
