@@ -32,12 +32,14 @@
 //   warp 10     scheduler: takes the next unit and prepares its metadata
 //               (page, rows, private lengths, fork limits, packed page ids)
 //               in one of two shared-memory slots while the other is in use.
-//   warps 0, 11 TMA producers: warp 0 the unit's K blocks, warp 11 its V
-//               blocks, each into a three-stage ring (128-byte swizzle); a K
-//               stage is refilled as soon as its Q K^T is done, whatever the
-//               V ring waits for.
-//   warp 1      TMEM owner and MMA issuer; one global sequence of blocks
-//               across units, in the order QK(b), PV(b-1):
+//   warps 0, 11 TMA producers: warp 0 the unit's Q tile and then its K
+//               blocks, warp 11 its V blocks, each into a three-stage ring
+//               (128-byte swizzle); a K stage is refilled as soon as its Q
+//               K^T (or Q copy) is done, whatever the V ring waits for.
+//   warp 1      TMEM owner and MMA issuer: copies each unit's Q tile from
+//               its K stage into TMEM (tcgen05.cp, double buffered by unit),
+//               then one global sequence of blocks across units, in the
+//               order QK(b), PV(b-1):
 //                 S = Q K^T   Q read from TMEM, K from shared memory; S into
 //                             TMEM (fp32, double buffered by block)
 //                 O += P V    P read from TMEM (bf16, written over S), V from
@@ -50,9 +52,8 @@
 //               halves of a row exchange their partial max through shared
 //               memory.  O is rescaled in TMEM only when a row's running
 //               max grows by more than 2^8; the stale max stays exact after
-//               the final normalisation.  They also copy each unit's Q rows
-//               from global memory into TMEM (double buffered by unit), the
-//               next unit's before the current unit's epilogue.
+//               the final normalisation.  At a unit change they only read
+//               the next unit's metadata before the epilogue.
 // One split: the unit writes the final bf16 output and lse.  Several splits:
 // it writes its normalised fp32 partial and lse for merge.cu.
 // All waits are bounded; a timeout sets HPD_DEVERR_TIMEOUT, every role
