@@ -78,16 +78,23 @@ def algorithmic_work(inp, V=VOCAB):
     kernel must move or compute no matter how it is written)."""
     m, Hq, Hkv, D = inp.m, inp.H_q, inp.H_kv, inp.D
     P = np.diff(inp.prefix_cu).astype(np.float64)
-    Bd = np.diff(inp.branch_cu).astype(np.float64)
+    Bd = np.diff(inp.branch_cu).astype(np.int64)
     L = inp.branch_len.astype(np.float64)
+    # prefix keys each branch sees (its fork-position length, else its page's)
+    Pb = np.repeat(P, Bd)
+    if inp.branch_prefix_len is not None:
+        Pb = np.minimum(Pb, inp.branch_prefix_len.astype(np.float64))
+    # per page, the prefix keys some branch of it sees (read once)
+    P_read = np.array([Pb[inp.branch_cu[d]:inp.branch_cu[d + 1]].max(initial=0.0)
+                       for d in range(inp.n_docs)])
     rows = inp.B * m
     q_bytes = rows * Hq * D * 2
-    prefix_kv = P.sum() * Hkv * D * 2 * 2
+    prefix_kv = P_read.sum() * Hkv * D * 2 * 2
     private_kv = L.sum() * Hkv * D * 2 * 2
     pages_used = np.ceil(L / W.PAGE).sum()
     tables = pages_used * 4 + inp.B * 4 + 2 * (inp.n_docs + 1) * 4
     out_bytes = rows * Hq * D * 2 + rows * Hq * 4
-    prefix_flops = 4.0 * (Bd * m * Hq * P).sum() * D
+    prefix_flops = 4.0 * m * Hq * D * Pb.sum()
     vis = np.zeros(inp.B)
     for i in range(m):
         vis += np.maximum(0.0, L - m + i + 1)
